@@ -1,0 +1,6 @@
+"""Seeded synthetic inputs shared by the tests, bench.py and the oracle's callers.
+
+This package holds shapes and random draws only: no step of the method
+(masking, ELBO, bound, gradient, advantage normalisation) is computed here.
+"""
+from .workloads import CONFIGS, Workload, make_inputs, zipf_targets  # noqa: F401

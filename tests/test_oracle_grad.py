@@ -1,0 +1,114 @@
+"""Pins of the oracle's analytic gradients (Algorithm 1 backward, Sec. 3.2 Equivalence)."""
+import numpy as np
+import torch
+
+from oracle import bgpo_oracle as O
+
+
+def _case(seed=0, B=3, P=2, R=9, H=6, V=23, n_t=3, t_mode=0, off_policy=True):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((B, P + R, H))
+    W = rng.standard_normal((V, H)) * 0.7
+    Y = rng.integers(0, V, size=(B, R))
+    A = rng.standard_normal(B)
+    A[0] = abs(A[0])            # both branches present
+    A[1] = -abs(A[1])
+    ts, masks = O.sample_masks(seed + 100, B, R, n_t, t_mode)
+    ell_self = O.elbo_all(X, W, Y, P, ts, masks)
+    eps = rng.standard_normal((B, n_t)) * 0.3 if off_policy else np.zeros((B, n_t))
+    ell_old = ell_self + eps
+    return X, W, Y, P, A, ell_old, ts, masks
+
+
+def _fd_check(loss_fn, X, W, dX, dW, P, n=25, h=1e-6, seed=0):
+    rng = np.random.default_rng(seed)
+    V, H = W.shape
+    B, R = dX.shape[:2]
+    for _ in range(n):
+        v, k = rng.integers(V), rng.integers(H)
+        Wp, Wm = W.copy(), W.copy()
+        Wp[v, k] += h
+        Wm[v, k] -= h
+        fd = (loss_fn(X, Wp) - loss_fn(X, Wm)) / (2 * h)
+        assert abs(fd - dW[v, k]) <= 1e-6 * max(1.0, abs(fd)), (v, k, fd, dW[v, k])
+    for _ in range(n):
+        b, i, k = rng.integers(B), rng.integers(R), rng.integers(H)
+        Xp, Xm = X.copy(), X.copy()
+        Xp[b, P + i, k] += h
+        Xm[b, P + i, k] -= h
+        fd = (loss_fn(Xp, W) - loss_fn(Xm, W)) / (2 * h)
+        assert abs(fd - dX[b, i, k]) <= 1e-6 * max(1.0, abs(fd)), (b, i, k, fd, dX[b, i, k])
+
+
+def test_gradients_match_finite_differences_off_policy():
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=1)
+    ls = 0.5
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, ls)
+    f = lambda X_, W_: O.bgpo_loss(X_, W_, Y, P, A, ell_old, ts, masks, ls)
+    _fd_check(f, X, W, out["dX"], out["dW"], P, seed=1)
+
+
+def test_gradients_match_finite_differences_stratified():
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=2, n_t=4, t_mode=1)
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, 1.0)
+    f = lambda X_, W_: O.bgpo_loss(X_, W_, Y, P, A, ell_old, ts, masks, 1.0)
+    _fd_check(f, X, W, out["dX"], out["dW"], P, seed=2)
+
+
+def test_gradients_match_torch_autograd():
+    # an independent statement of the same loss, differentiated by torch autograd
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=3, B=4, R=12, H=10, V=40, n_t=5)
+    ls = 0.25
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, ls)
+    Xt = torch.tensor(X, requires_grad=True)
+    Wt = torch.tensor(W, requires_grad=True)
+    n_t = len(ts)
+    total = torch.zeros((), dtype=torch.float64)
+    for j in range(n_t):
+        for b in range(X.shape[0]):
+            m = torch.from_numpy(masks[j, b].astype(bool))
+            resp = Xt[b, P:]
+            lp = torch.log_softmax(resp @ Wt.T, dim=1).gather(1, torch.from_numpy(Y[b]).long()[:, None])[:, 0]
+            ell = (lp * m).sum() / float(ts[j, b])
+            d = ell - float(ell_old[b, j])
+            g = (1 + d) * A[b] / n_t if A[b] >= 0 else torch.exp(d) * A[b] / n_t
+            total = total - ls * g
+    total.backward()
+    assert abs(float(total.detach()) - out["loss"]) < 1e-10 * max(1, abs(out["loss"]))
+    assert np.allclose(Wt.grad.numpy(), out["dW"], rtol=1e-10, atol=1e-12)
+    assert np.allclose(Xt.grad[:, P:].numpy(), out["dX"], rtol=1e-10, atol=1e-12)
+    assert np.array_equal(Xt.grad[:, :P].numpy(), np.zeros_like(Xt.grad[:, :P].numpy()))
+
+
+def test_equivalence_gradient_on_policy():
+    # Sec. 3.2: on-policy, grad R_lb = grad R_hat; R_hat (Eq. 7) differentiated numerically
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=4, off_policy=False)
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, 1.0)
+    assert np.allclose(out["d"], 0.0, atol=0)
+    assert np.allclose(out["R_lb"], A, rtol=1e-13)
+    f = lambda X_, W_: O.vrpo_loss(X_, W_, Y, P, A, ell_old, ts, masks, 1.0)
+    _fd_check(f, X, W, out["dX"], out["dW"], P, seed=4)
+
+
+def test_dw_rows_sum_to_zero():
+    # each dz_r = w_r (onehot - softmax) sums to zero over the vocabulary
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=5, V=57)
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, 1.0)
+    scale = np.abs(out["dW"]).max()
+    assert np.abs(out["dW"].sum(axis=0)).max() < 1e-12 * max(1.0, scale)
+
+
+def test_linearity_accumulation_equals_one_shot():
+    # Linearity (Sec. 3): summing per-sample gradients = gradient of sum_j L_j;
+    # here the per-sample pieces are accumulated in reverse order and in halves
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=6, n_t=6)
+    out = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, 1.0)
+    coef = out["coef"]
+    dW = np.zeros_like(W)
+    dX = np.zeros_like(out["dX"])
+    for j in reversed(range(6)):
+        gx, gw = O.elbo_term_grads(X, W, Y, P, masks[j], ts[j], coef[:, j], chunk=5)
+        dX += gx
+        dW += gw
+    assert np.allclose(dW, out["dW"], rtol=1e-12, atol=1e-14)
+    assert np.allclose(dX, out["dX"], rtol=1e-12, atol=1e-14)
