@@ -1,0 +1,231 @@
+/*
+ * bgpo.h -- C ABI of the GB300 (sm_103a) BGPO masked-diffusion ELBO hot path.
+ *
+ * Boundary-Guided Policy Optimization (arxiv 2510.11683) trains a diffusion LLM
+ * on a linear lower bound of its ELBO-based RL objective. Per Monte Carlo sample
+ * j of each response b the path is:
+ *
+ *   bgpo_sample_mask          t_{b,j} and the response mask (Sec. 2.1; Eq. 3, 5;
+ *                             Algorithm 1, sampling of t and y_t)
+ *   bgpo_elbo_fwd             l_{b,j} = (1/t) sum_masked log p(y^i | y_t, x) through
+ *                             the LM head (Eq. 4), full logits never stored
+ *   bgpo_bound_coeffs         d_j (Eq. 10), g_j (Eq. 13) and dL_j/dl_j with
+ *                             L_j = -loss_scale * g_j (Algorithm 1; Eq. 19)
+ *   bgpo_elbo_bwd_accumulate  dX += dL_j/dX, dW += dL_j/dW (Algorithm 1, gradient
+ *                             accumulation; Linearity, Sec. 3), so memory does
+ *                             not grow with n_t
+ *
+ * plus bgpo_group_advantage (Eq. 18).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Pointers marked "device" are CUDA device pointers on the current device;
+ *    "host" pointers are ordinary host memory. The caller allocates and owns
+ *    every buffer, including one workspace of bgpo_workspace_bytes() bytes.
+ *    The library allocates no device memory.
+ *  - All launches are asynchronous on `stream` (a cudaStream_t; NULL = the
+ *    legacy default stream). No call synchronises except
+ *    bgpo_get_device_error and bgpo_trace_get.
+ *  - Dtypes are fixed: X and W bfloat16, Y int32, everything else float32.
+ *  - Layouts are dense row-major: X [B, P+R, H], W [V, H], Y [B, R],
+ *    dX [B, R, H] (response rows only), dW [V, H], per-sequence vectors [B].
+ *  - Alignment: X, W, dX, dW and the workspace must be 16-byte aligned
+ *    (workspace: 256-byte). H must be a multiple of 64.
+ *  - The workspace carries sample j's draws (t, mask), its compacted masked
+ *    rows and forward statistics from one call to the next, so the calls for
+ *    one sample must be issued in the order
+ *        bgpo_sample_mask -> bgpo_elbo_fwd -> [bgpo_bound_coeffs] ->
+ *        bgpo_elbo_bwd_accumulate
+ *    on one stream, with the same j. A call made with a j other than the one
+ *    the workspace holds sets the device error word to BGPO_ERR_INVALID_ARG
+ *    and does no work.
+ *  - Host-side checks return a status before anything is launched. A failed
+ *    launch returns BGPO_ERR_CUDA. Faults detected on the device (a non-finite
+ *    coefficient, a bounded wait that ran out, a sample mismatch) are recorded
+ *    in an error word inside the workspace: read it with bgpo_get_device_error.
+ *  - The device must have compute capability 10.3 (GB300); otherwise every
+ *    launching call returns BGPO_ERR_UNSUPPORTED_DEVICE.
+ */
+#ifndef BGPO_H_
+#define BGPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BGPO_ABI_VERSION 1
+
+typedef enum bgpo_status {
+  BGPO_OK = 0,
+  BGPO_ERR_INVALID_ARG = 1,          /* null pointer, j out of range, bad enum */
+  BGPO_ERR_SHAPE = 2,                /* sizes out of the supported range */
+  BGPO_ERR_ALIGNMENT = 3,            /* pointer not aligned as required */
+  BGPO_ERR_WORKSPACE_TOO_SMALL = 4,  /* ws_bytes < bgpo_workspace_bytes() */
+  BGPO_ERR_NONFINITE = 5,            /* non-finite bound coefficient (device) */
+  BGPO_ERR_UNSUPPORTED_DEVICE = 6,   /* current device is not sm_103 */
+  BGPO_ERR_CUDA = 7,                 /* a CUDA runtime call or launch failed */
+  BGPO_ERR_TIMEOUT = 8               /* a bounded device-side wait ran out */
+} bgpo_status;
+
+/* Optional per-kernel timing: CUDA events recorded around each kernel launch. */
+typedef struct bgpo_trace bgpo_trace;
+
+/* t_mode values */
+#define BGPO_T_IID 0         /* t_{b,j} i.i.d. on (0, 1] (Eq. 5) */
+#define BGPO_T_STRATIFIED 1  /* t_{b,j} in (j/n_t, (j+1)/n_t]; not in the paper */
+
+/*
+ * Problem description (host struct, read by every call; never stored).
+ *   B      responses in the batch (>= 1)
+ *   P      prompt length: X rows [b, 0, P) are the prompt, never masked (Sec. 2.1)
+ *   R      response length (>= 1); response position i is X row [b, P + i]
+ *   H      hidden size, multiple of 64, 64 <= H <= 16384
+ *   V      vocabulary size, 1 <= V <= 2^24
+ *   n_t    MC samples per response, 1 <= n_t < 65536 (Eq. 5)
+ *   G      group size used by bgpo_group_advantage (Eq. 18), >= 1
+ *   t_mode BGPO_T_IID or BGPO_T_STRATIFIED
+ *   seed   Philox4x64-10 key word 0; the draws of (b, j) depend on (seed, b, j) only
+ *   loss_scale  L_j = -loss_scale * g_j; Algorithm 1 uses 1/G
+ *   trace  optional bgpo_trace* (NULL = off)
+ * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
+ * bgpo_workspace_bytes).
+ */
+typedef struct bgpo_problem {
+  int32_t B;
+  int32_t P;
+  int32_t R;
+  int32_t H;
+  int32_t V;
+  int32_t n_t;
+  int32_t G;
+  int32_t t_mode;
+  uint64_t seed;
+  float loss_scale;
+  int32_t flags;       /* reserved, must be 0 */
+  bgpo_trace* trace;
+} bgpo_problem;
+
+/* ABI version of the loaded library (BGPO_ABI_VERSION). */
+int32_t bgpo_abi_version(void);
+
+/* Human-readable name of a status code (static string). */
+const char* bgpo_status_string(bgpo_status status);
+
+/*
+ * Host-only validation of a problem description (no CUDA call).
+ * Returns BGPO_OK, BGPO_ERR_INVALID_ARG (NULL, bad t_mode, flags != 0,
+ * non-finite loss_scale) or BGPO_ERR_SHAPE.
+ */
+bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
+
+/*
+ * Bytes of device workspace the calls below need for `prob`. Depends on B, R,
+ * H and V only -- never on n_t (Linearity, Sec. 3: one sample's state at a
+ * time). Returns 0 for an invalid problem.
+ */
+size_t bgpo_workspace_bytes(const bgpo_problem* prob);
+
+/*
+ * Forward masking process for MC sample j (Sec. 2.1; Eq. 3, 5; Algorithm 1).
+ * Draws t_{b,j} = T/D with Philox4x64-10 (key (seed, 0), counter (0, b, j, 1),
+ * T = u24 + 1 and D = 2^24, or T = j 2^24 + u24 + 1 and D = n_t 2^24 when
+ * stratified; u24 = top 24 bits of output word 0) and masks response position
+ * i of sequence b iff u24_i * D < T * 2^24, where u24_i is the top 24 bits of
+ * output word (i mod 4) of the block with counter (i / 4, b, j, 0). Prompt
+ * positions are never masked. Compacts the masked positions into ascending
+ * (b, i) order inside the workspace.
+ *   j         sample index, 0 <= j < n_t
+ *   ws        device workspace (256-byte aligned), ws_bytes its size
+ *   t_out     device float [B] or NULL: t_{b,j} rounded to float
+ *   mask_out  device uint8 [B, R] or NULL: 1 = masked
+ */
+bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size_t ws_bytes,
+                             float* t_out, uint8_t* mask_out, void* stream);
+
+/*
+ * Per-step ELBO term of Eq. 4 for sample j, every sequence:
+ *   l_{b,j} = (1 / t_{b,j}) * sum_{i masked} log softmax(W x_{b,P+i})[Y[b,i]]
+ * (no length normalisation; an empty mask gives 0). The masked rows of X are
+ * gathered, multiplied by W on the tensor cores (bf16 in, fp32 accumulate)
+ * and reduced by an online log-sum-exp per row; the per-row log-sum-exp and
+ * log-probabilities stay in the workspace for the backward pass. The result is
+ * deterministic (fixed reduction order), so recomputing l with unchanged inputs
+ * gives bit-identical values (on-policy d_j = 0 exactly, Sec. 3.2).
+ *   X      device bf16 [B, P+R, H];  W device bf16 [V, H];  Y device int32 [B, R]
+ *          with 0 <= Y < V (out-of-range targets give an undefined l)
+ *   ell_out device float [B]: l_{b,j} (e.g. column j of a [n_t, B] array)
+ * Requires a preceding bgpo_sample_mask(j) on the same workspace.
+ */
+bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, const void* W,
+                          const int32_t* Y, void* ws, size_t ws_bytes, float* ell_out,
+                          void* stream);
+
+/*
+ * BGPO bound coefficients for sample j (Eq. 10, 13; Algorithm 1; Eq. 19):
+ *   d     = ell - ell_old                       (same t and mask for both policies)
+ *   g     = (1 + d) A / n_t        if A >= 0    (Lemma 1, Taylor)
+ *           e^d A / n_t            if A <  0    (Lemma 2, Jensen)
+ *   coef  = dL_j / dl_j = -loss_scale * A * (A >= 0 ? 1 : e^d) / n_t
+ * All pointers device float [B]. g_out may be NULL. A non-finite g or coef
+ * sets the device error word to BGPO_ERR_NONFINITE (values are still written).
+ */
+bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* ell,
+                              const float* ell_old, const float* A, float* coef_out, float* g_out,
+                              void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Backward pass of L_j = sum_b coef_b * l_{b,j}, accumulated (Algorithm 1,
+ * gradient accumulation; Eq. 15-17 give the per-sample gradient weights):
+ *   w_r   = coef_b / t_{b,j}                       for masked row r = (b, i)
+ *   dz_r  = w_r (onehot(Y[b,i]) - softmax(W x_r))  (logits recomputed; bf16)
+ *   dX[b, i, :] += W^T dz_r        dW += sum_r dz_r x_r^T
+ * coef is an input (normally bgpo_bound_coeffs' output for the same j).
+ *   dX device float [B, R, H], dW device float [V, H]: accumulated in place.
+ * Deterministic: no atomics, fixed summation order.
+ * Requires bgpo_sample_mask(j) and bgpo_elbo_fwd(j) before it on the same
+ * workspace, with the same X, W and Y.
+ */
+bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
+                                     const void* W, const int32_t* Y, const float* coef, void* ws,
+                                     size_t ws_bytes, float* dX, float* dW, void* stream);
+
+/*
+ * Group-normalised advantages (Eq. 18) over consecutive groups of G responses:
+ *   A = (r - mean_G r) / std_G r, population std; a zero-std group gets A = 0.
+ *   rewards, A_out: device float [B]; B must be a multiple of G.
+ */
+bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards, float* A_out,
+                                 void* stream);
+
+/*
+ * Reads the device error word of a workspace (synchronises `stream`).
+ *   code_out: BGPO_OK or the first device-detected status; where_out (may be
+ *   NULL): kernel and site that set it.
+ */
+bgpo_status bgpo_get_device_error(const void* ws, size_t ws_bytes, int32_t* code_out,
+                                  int32_t* where_out, void* stream);
+
+/* Clears the device error word (asynchronous on `stream`). */
+bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream);
+
+/* ---- per-kernel timing (host objects holding CUDA events) ---------------- */
+
+/* Creates a trace that can hold `capacity` kernel launches; NULL on failure. */
+bgpo_trace* bgpo_trace_create(int32_t capacity);
+void bgpo_trace_destroy(bgpo_trace* trace);
+/* Forgets recorded launches (events are reused). */
+void bgpo_trace_reset(bgpo_trace* trace);
+int32_t bgpo_trace_count(const bgpo_trace* trace);
+/* Kernel id and duration in ms of recorded launch idx (waits for it). */
+bgpo_status bgpo_trace_get(const bgpo_trace* trace, int32_t idx, int32_t* kernel_id, float* ms);
+/* Name of a kernel id (static string), "?" if unknown. */
+const char* bgpo_kernel_name(int32_t kernel_id);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BGPO_H_ */

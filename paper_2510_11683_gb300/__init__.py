@@ -1,0 +1,185 @@
+"""GB300-native BGPO masked-diffusion ELBO hot path (arxiv 2510.11683).
+
+Thin PyTorch binding over the C ABI of ``include/bgpo.h``. Every step of the
+path runs in the CUDA kernels of ``lib/libbgpo.so``; this module only checks
+tensor dtypes/devices and passes raw pointers and the current CUDA stream.
+
+Per MC sample j (Algorithm 1):
+
+    sample_mask(prob, j, ws)                       # t_{b,j}, mask (Sec. 2.1)
+    elbo_fwd(prob, j, X, W, Y, ws, ell[j])         # Eq. 4 through the LM head
+    bound_coeffs(prob, j, ell[j], ell_old[j], A, coef, g, ws)   # Eq. 10, 13
+    elbo_bwd_accumulate(prob, j, X, W, Y, coef, ws, dX, dW)     # dX, dW +=
+"""
+import ctypes
+
+from . import _lib
+from ._lib import BgpoError, BgpoProblem  # noqa: F401
+
+T_IID = 0
+T_STRATIFIED = 1
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None):
+    """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1)."""
+    p = BgpoProblem()
+    p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
+    p.seed = seed
+    p.loss_scale = (1.0 / G if G > 0 else 1.0) if loss_scale is None else loss_scale
+    p.flags = 0
+    p.trace = trace.handle if isinstance(trace, Trace) else trace
+    return p
+
+
+def problem_from(wl, trace=None, loss_scale=None):
+    """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
+    return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
+                   loss_scale=loss_scale, trace=trace)
+
+
+def validate_problem(prob):
+    return _lib.lib().bgpo_validate_problem(ctypes.byref(prob))
+
+
+def workspace_bytes(prob):
+    n = _lib.lib().bgpo_workspace_bytes(ctypes.byref(prob))
+    if n == 0:
+        raise BgpoError("bgpo_workspace_bytes", validate_problem(prob))
+    return n
+
+
+def alloc_workspace(prob, device="cuda"):
+    """A uint8 device tensor of workspace_bytes(prob) (256-byte aligned by torch)."""
+    torch = _torch()
+    ws = torch.empty(workspace_bytes(prob), dtype=torch.uint8, device=device)
+    assert ws.data_ptr() % 256 == 0
+    return ws
+
+
+def _ptr(t, dtype=None, name="tensor"):
+    if t is None:
+        return None
+    torch = _torch()
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    torch = _torch()
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def sample_mask(prob, j, ws, t_out=None, mask_out=None, stream=None):
+    torch = _torch()
+    st = _lib.lib().bgpo_sample_mask(
+        ctypes.byref(prob), j, _ptr(ws, torch.uint8, "ws"), ws.numel(),
+        _ptr(t_out, torch.float32, "t_out"), _ptr(mask_out, torch.uint8, "mask_out"),
+        _stream(stream))
+    _lib.check("bgpo_sample_mask", st)
+
+
+def elbo_fwd(prob, j, X, W, Y, ws, ell_out, stream=None):
+    torch = _torch()
+    st = _lib.lib().bgpo_elbo_fwd(
+        ctypes.byref(prob), j, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(Y, torch.int32, "Y"), _ptr(ws, torch.uint8, "ws"), ws.numel(),
+        _ptr(ell_out, torch.float32, "ell_out"), _stream(stream))
+    _lib.check("bgpo_elbo_fwd", st)
+
+
+def bound_coeffs(prob, j, ell, ell_old, A, coef_out, g_out, ws, stream=None):
+    torch = _torch()
+    f32 = torch.float32
+    st = _lib.lib().bgpo_bound_coeffs(
+        ctypes.byref(prob), j, _ptr(ell, f32, "ell"), _ptr(ell_old, f32, "ell_old"),
+        _ptr(A, f32, "A"), _ptr(coef_out, f32, "coef_out"), _ptr(g_out, f32, "g_out"),
+        _ptr(ws, torch.uint8, "ws"), ws.numel(), _stream(stream))
+    _lib.check("bgpo_bound_coeffs", st)
+
+
+def elbo_bwd_accumulate(prob, j, X, W, Y, coef, ws, dX, dW, stream=None):
+    torch = _torch()
+    f32 = torch.float32
+    st = _lib.lib().bgpo_elbo_bwd_accumulate(
+        ctypes.byref(prob), j, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(Y, torch.int32, "Y"), _ptr(coef, f32, "coef"), _ptr(ws, torch.uint8, "ws"),
+        ws.numel(), _ptr(dX, f32, "dX"), _ptr(dW, f32, "dW"), _stream(stream))
+    _lib.check("bgpo_elbo_bwd_accumulate", st)
+
+
+def group_advantage(prob, rewards, A_out, stream=None):
+    torch = _torch()
+    st = _lib.lib().bgpo_group_advantage(
+        ctypes.byref(prob), _ptr(rewards, torch.float32, "rewards"),
+        _ptr(A_out, torch.float32, "A_out"), _stream(stream))
+    _lib.check("bgpo_group_advantage", st)
+
+
+def get_device_error(ws, stream=None):
+    """(status, where) of the workspace's device error word (synchronises)."""
+    torch = _torch()
+    code = ctypes.c_int32(0)
+    where = ctypes.c_int32(0)
+    st = _lib.lib().bgpo_get_device_error(_ptr(ws, torch.uint8, "ws"), ws.numel(),
+                                          ctypes.byref(code), ctypes.byref(where), _stream(stream))
+    _lib.check("bgpo_get_device_error", st)
+    return code.value, where.value
+
+
+def clear_device_error(ws, stream=None):
+    torch = _torch()
+    st = _lib.lib().bgpo_clear_device_error(_ptr(ws, torch.uint8, "ws"), ws.numel(),
+                                            _stream(stream))
+    _lib.check("bgpo_clear_device_error", st)
+
+
+def kernel_name(kid):
+    return _lib.lib().bgpo_kernel_name(kid).decode()
+
+
+class Trace:
+    """Per-kernel CUDA-event timing: pass ``trace=`` to ``problem``."""
+
+    def __init__(self, capacity):
+        self.handle = _lib.lib().bgpo_trace_create(capacity)
+        if not self.handle:
+            raise BgpoError("bgpo_trace_create", 7)
+
+    def reset(self):
+        _lib.lib().bgpo_trace_reset(self.handle)
+
+    def records(self):
+        """[(kernel name, ms)] of the launches recorded since the last reset."""
+        L = _lib.lib()
+        out = []
+        for i in range(L.bgpo_trace_count(self.handle)):
+            kid = ctypes.c_int32(0)
+            ms = ctypes.c_float(0)
+            _lib.check("bgpo_trace_get", L.bgpo_trace_get(self.handle, i, ctypes.byref(kid),
+                                                          ctypes.byref(ms)))
+            out.append((kernel_name(kid.value), ms.value))
+        return out
+
+    def close(self):
+        if self.handle:
+            _lib.lib().bgpo_trace_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

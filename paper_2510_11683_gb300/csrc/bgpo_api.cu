@@ -1,0 +1,401 @@
+// Host side of the C ABI declared in include/bgpo.h: argument validation,
+// workspace layout, TMA tensor-map encoding, kernel launches and per-kernel
+// event tracing. Keeps no state between calls except the cached driver entry
+// point of cuTensorMapEncodeTiled.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "bgpo.h"
+#include "bgpo_internal.h"
+#include "bgpo_plan.h"
+
+using namespace bgpo;
+
+struct bgpo_trace {
+  int32_t capacity;
+  int32_t count;
+  int32_t* ids;
+  cudaEvent_t* start;
+  cudaEvent_t* stop;
+};
+
+namespace {
+
+constexpr int64_t kMaxRows = int64_t(1) << 22;  // B * R
+constexpr int64_t kMaxV = int64_t(1) << 24;
+constexpr int64_t kMaxH = 16384;
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Records CUDA events around one kernel launch when a trace is attached.
+struct TraceScope {
+  bgpo_trace* tr;
+  cudaStream_t s;
+  int32_t idx;
+  TraceScope(bgpo_trace* t, int32_t kid, cudaStream_t st) : tr(t), s(st), idx(-1) {
+    if (tr && tr->count < tr->capacity) {
+      idx = tr->count++;
+      tr->ids[idx] = kid;
+      cudaEventRecord(tr->start[idx], s);
+    }
+  }
+  ~TraceScope() {
+    if (idx >= 0) cudaEventRecord(tr->stop[idx], s);
+  }
+};
+
+bgpo_status check_problem(const bgpo_problem* p) {
+  if (!p) return BGPO_ERR_INVALID_ARG;
+  if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
+  if (p->flags != 0) return BGPO_ERR_INVALID_ARG;
+  if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
+  if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
+  if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
+  if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
+  if ((int64_t)p->B * p->R > kMaxRows) return BGPO_ERR_SHAPE;
+  if ((int64_t)p->B * ((int64_t)p->P + p->R) * p->H > (int64_t(1) << 40)) return BGPO_ERR_SHAPE;
+  return BGPO_OK;
+}
+
+Geometry geometry_of(const bgpo_problem* p) { return make_geometry(p->B, p->P, p->R, p->H, p->V); }
+
+bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
+  return (j >= 0 && j < p->n_t) ? BGPO_OK : BGPO_ERR_INVALID_ARG;
+}
+
+bgpo_status check_ws(const bgpo_problem* p, const void* ws, size_t ws_bytes, WsLayout* L) {
+  if (!ws) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
+  *L = make_ws_layout(geometry_of(p));
+  if (ws_bytes < L->total) return BGPO_ERR_WORKSPACE_TOO_SMALL;
+  return BGPO_OK;
+}
+
+bgpo_status device_sms(int* num_sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return BGPO_ERR_UNSUPPORTED_DEVICE;
+  }
+  int major = 0, minor = 0, sms = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return BGPO_ERR_CUDA;
+  }
+  if (major != 10 || minor != 3) return BGPO_ERR_UNSUPPORTED_DEVICE;
+  *num_sms = sms;
+  return BGPO_OK;
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+    else
+      cudaGetLastError();
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [outer, inner] matrix with row pitch
+// `pitch_bytes`, 128-byte swizzle, zero fill outside the matrix.
+bool map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+            uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn enc = encode_tiled();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {pitch_bytes};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bgpo_status from_cuda(cudaError_t e) { return e == cudaSuccess ? BGPO_OK : BGPO_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t bgpo_abi_version(void) { return BGPO_ABI_VERSION; }
+
+const char* bgpo_status_string(bgpo_status s) {
+  switch (s) {
+    case BGPO_OK: return "BGPO_OK";
+    case BGPO_ERR_INVALID_ARG: return "BGPO_ERR_INVALID_ARG";
+    case BGPO_ERR_SHAPE: return "BGPO_ERR_SHAPE";
+    case BGPO_ERR_ALIGNMENT: return "BGPO_ERR_ALIGNMENT";
+    case BGPO_ERR_WORKSPACE_TOO_SMALL: return "BGPO_ERR_WORKSPACE_TOO_SMALL";
+    case BGPO_ERR_NONFINITE: return "BGPO_ERR_NONFINITE";
+    case BGPO_ERR_UNSUPPORTED_DEVICE: return "BGPO_ERR_UNSUPPORTED_DEVICE";
+    case BGPO_ERR_CUDA: return "BGPO_ERR_CUDA";
+    case BGPO_ERR_TIMEOUT: return "BGPO_ERR_TIMEOUT";
+  }
+  return "BGPO_ERR_UNKNOWN";
+}
+
+bgpo_status bgpo_validate_problem(const bgpo_problem* prob) { return check_problem(prob); }
+
+size_t bgpo_workspace_bytes(const bgpo_problem* prob) {
+  if (check_problem(prob) != BGPO_OK) return 0;
+  return make_ws_layout(geometry_of(prob)).total;
+}
+
+bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size_t ws_bytes,
+                             float* t_out, uint8_t* mask_out, void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if ((st = check_sample(prob, j)) != BGPO_OK) return st;
+  WsLayout L;
+  if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
+  if (t_out && !aligned(t_out, 4)) return BGPO_ERR_ALIGNMENT;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const WsPtrs w = ws_pointers(ws, L);
+  MaskArgs a;
+  a.seed = prob->seed;
+  a.B = prob->B;
+  a.R = prob->R;
+  a.j = j;
+  a.n_t = prob->n_t;
+  a.t_mode = prob->t_mode;
+  a.t_out = t_out;
+  a.mask_out = mask_out;
+  TraceScope ts(prob->trace, KID_MASK_COMPACT, s);
+  return from_cuda(launch_mask_compact(a, w, s));
+}
+
+bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, const void* W,
+                          const int32_t* Y, void* ws, size_t ws_bytes, float* ell_out,
+                          void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if ((st = check_sample(prob, j)) != BGPO_OK) return st;
+  if (!X || !W || !Y || !ell_out) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 4) || !aligned(ell_out, 4))
+    return BGPO_ERR_ALIGNMENT;
+  WsLayout L;
+  if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Geometry g = geometry_of(prob);
+  const WsPtrs w = ws_pointers(ws, L);
+
+  CUtensorMap map_xm, map_w;
+  if (!map_2d(&map_xm, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
+      !map_2d(&map_w, W, g.H, g.V, g.H * 2, kBK, kBN))
+    return BGPO_ERR_CUDA;
+  GemmArgs ga;
+  ga.g = g;
+  ga.num_sms = sms;
+  ga.j = j;
+  ga.coef = nullptr;
+  ga.dW = nullptr;
+  {
+    TraceScope ts(prob->trace, KID_GATHER, s);
+    if (launch_gather(g, j, X, Y, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_LMHEAD_FWD, s);
+    if (launch_gemm(GEMM_FWD, map_xm, map_w, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_LSE_COMBINE, s);
+    if (launch_lse_combine(g, j, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_SEQ_REDUCE, s);
+    if (launch_seq_reduce(g, j, w, ell_out, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  return BGPO_OK;
+}
+
+bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* ell,
+                              const float* ell_old, const float* A, float* coef_out, float* g_out,
+                              void* ws, size_t ws_bytes, void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if ((st = check_sample(prob, j)) != BGPO_OK) return st;
+  if (!ell || !ell_old || !A || !coef_out) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ell, 4) || !aligned(ell_old, 4) || !aligned(A, 4) || !aligned(coef_out, 4) ||
+      (g_out && !aligned(g_out, 4)))
+    return BGPO_ERR_ALIGNMENT;
+  WsLayout L;
+  if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const WsPtrs w = ws_pointers(ws, L);
+  TraceScope ts(prob->trace, KID_BOUND_COEFFS, s);
+  return from_cuda(launch_bound_coeffs(prob->B, prob->n_t, prob->loss_scale, ell, ell_old, A,
+                                       coef_out, g_out, w, s));
+}
+
+bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
+                                     const void* W, const int32_t* Y, const float* coef, void* ws,
+                                     size_t ws_bytes, float* dX, float* dW, void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if ((st = check_sample(prob, j)) != BGPO_OK) return st;
+  if (!X || !W || !Y || !coef || !dX || !dW) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 4) || !aligned(coef, 4) ||
+      !aligned(dX, 16) || !aligned(dW, 16))
+    return BGPO_ERR_ALIGNMENT;
+  WsLayout L;
+  if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Geometry g = geometry_of(prob);
+  const WsPtrs w = ws_pointers(ws, L);
+
+  CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xm_mn;
+  if (!map_2d(&map_xm_k, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
+      !map_2d(&map_w_k, W, g.H, g.V, g.H * 2, kBK, kBN) ||
+      !map_2d(&map_dz_k, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, kBK, kBM) ||
+      !map_2d(&map_w_mn, W, g.H, g.V, g.H * 2, 64, kBK) ||
+      !map_2d(&map_dz_mn, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, kBK) ||
+      !map_2d(&map_xm_mn, w.xm, g.H, g.m_pad, g.H * 2, 64, kBK))
+    return BGPO_ERR_CUDA;
+  GemmArgs ga;
+  ga.g = g;
+  ga.num_sms = sms;
+  ga.j = j;
+  ga.coef = coef;
+  ga.dW = dW;
+  {
+    TraceScope ts(prob->trace, KID_LMHEAD_DZ, s);
+    if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_DX_GEMM, s);
+    if (launch_gemm(GEMM_DX, map_dz_k, map_w_mn, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_DX_REDUCE, s);
+    if (launch_dx_reduce(g, j, sms, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
+    TraceScope ts(prob->trace, KID_DW_GEMM, s);
+    if (launch_gemm(GEMM_DW, map_dz_mn, map_xm_mn, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  return BGPO_OK;
+}
+
+bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards, float* A_out,
+                                 void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if (!rewards || !A_out) return BGPO_ERR_INVALID_ARG;
+  if (prob->B % prob->G != 0) return BGPO_ERR_SHAPE;
+  if (!aligned(rewards, 4) || !aligned(A_out, 4)) return BGPO_ERR_ALIGNMENT;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  TraceScope ts(prob->trace, KID_GROUP_ADV, s);
+  return from_cuda(launch_group_advantage(prob->B, prob->G, rewards, A_out, s));
+}
+
+bgpo_status bgpo_get_device_error(const void* ws, size_t ws_bytes, int32_t* code_out,
+                                  int32_t* where_out, void* stream) {
+  if (!ws || !code_out) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
+  if (ws_bytes < 64) return BGPO_ERR_WORKSPACE_TOO_SMALL;
+  int32_t host[2] = {0, 0};
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(host, ws, sizeof(host), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return BGPO_ERR_CUDA;
+  }
+  *code_out = host[ERR_STATUS];
+  if (where_out) *where_out = host[ERR_WHERE];
+  return BGPO_OK;
+}
+
+bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream) {
+  if (!ws) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
+  if (ws_bytes < 64) return BGPO_ERR_WORKSPACE_TOO_SMALL;
+  return from_cuda(cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), static_cast<cudaStream_t>(stream)));
+}
+
+bgpo_trace* bgpo_trace_create(int32_t capacity) {
+  if (capacity <= 0) return nullptr;
+  bgpo_trace* t = static_cast<bgpo_trace*>(calloc(1, sizeof(bgpo_trace)));
+  if (!t) return nullptr;
+  t->capacity = capacity;
+  t->ids = static_cast<int32_t*>(calloc((size_t)capacity, sizeof(int32_t)));
+  t->start = static_cast<cudaEvent_t*>(calloc((size_t)capacity, sizeof(cudaEvent_t)));
+  t->stop = static_cast<cudaEvent_t*>(calloc((size_t)capacity, sizeof(cudaEvent_t)));
+  bool ok = t->ids && t->start && t->stop;
+  for (int32_t i = 0; ok && i < capacity; ++i)
+    ok = cudaEventCreate(&t->start[i]) == cudaSuccess && cudaEventCreate(&t->stop[i]) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    bgpo_trace_destroy(t);
+    return nullptr;
+  }
+  return t;
+}
+
+void bgpo_trace_destroy(bgpo_trace* t) {
+  if (!t) return;
+  for (int32_t i = 0; i < t->capacity; ++i) {
+    if (t->start && t->start[i]) cudaEventDestroy(t->start[i]);
+    if (t->stop && t->stop[i]) cudaEventDestroy(t->stop[i]);
+  }
+  free(t->ids);
+  free(t->start);
+  free(t->stop);
+  free(t);
+}
+
+void bgpo_trace_reset(bgpo_trace* t) {
+  if (t) t->count = 0;
+}
+
+int32_t bgpo_trace_count(const bgpo_trace* t) { return t ? t->count : 0; }
+
+bgpo_status bgpo_trace_get(const bgpo_trace* t, int32_t idx, int32_t* kernel_id, float* ms) {
+  if (!t || !kernel_id || !ms || idx < 0 || idx >= t->count) return BGPO_ERR_INVALID_ARG;
+  if (cudaEventSynchronize(t->stop[idx]) != cudaSuccess ||
+      cudaEventElapsedTime(ms, t->start[idx], t->stop[idx]) != cudaSuccess) {
+    cudaGetLastError();
+    return BGPO_ERR_CUDA;
+  }
+  *kernel_id = t->ids[idx];
+  return BGPO_OK;
+}
+
+const char* bgpo_kernel_name(int32_t id) {
+  static const char* names[KID_COUNT] = {
+      "mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
+      "bound_coeffs", "lmhead_dz",   "dx_gemm",        "dx_reduce",   "dw_gemm",
+      "group_advantage"};
+  return (id >= 0 && id < KID_COUNT) ? names[id] : "?";
+}
+
+}  // extern "C"

@@ -1,0 +1,66 @@
+// Launch interfaces between the C-ABI host code and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "bgpo_plan.h"
+
+namespace bgpo {
+
+// Pointers into one workspace (see WsLayout).
+struct WsPtrs {
+  int32_t* err;
+  float* t;
+  uint32_t* tnum;    // T numerators as (low, high) 32-bit pairs
+  int32_t* seg_off;
+  int32_t* rows;
+  int32_t* tgt;
+  float* tgt_logit;
+  float* lse;
+  float* logp;
+  float2* part;
+  void* xm;   // bf16
+  void* dz;   // bf16
+  float* dxp;
+};
+
+WsPtrs ws_pointers(void* ws, const WsLayout& L);
+
+struct MaskArgs {
+  uint64_t seed;
+  int32_t B, R, j, n_t, t_mode;
+  float* t_out;       // may be null
+  uint8_t* mask_out;  // may be null
+};
+
+cudaError_t launch_mask_compact(const MaskArgs& a, const WsPtrs& w, cudaStream_t s);
+cudaError_t launch_gather(const Geometry& g, int32_t j, const void* X, const int32_t* Y,
+                          const WsPtrs& w, cudaStream_t s);
+cudaError_t launch_lse_combine(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s);
+cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* ell_out,
+                              cudaStream_t s);
+cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
+                                const float* ell_old, const float* A, float* coef_out,
+                                float* g_out, const WsPtrs& w, cudaStream_t s);
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_sms, const WsPtrs& w,
+                             float* dX, cudaStream_t s);
+cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
+                                   cudaStream_t s);
+
+// The four tcgen05 GEMMs of the path.
+enum GemmKind : int { GEMM_FWD = 0, GEMM_DZ = 1, GEMM_DX = 2, GEMM_DW = 3 };
+
+struct GemmArgs {
+  Geometry g;
+  int num_sms;
+  int32_t j;
+  const float* coef;  // GEMM_DZ: per-sequence dL/dl
+  float* dW;          // GEMM_DW: accumulated weight gradient [V, H]
+};
+
+cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorMap& map_b,
+                        const GemmArgs& a, const WsPtrs& w, cudaStream_t s);
+
+}  // namespace bgpo

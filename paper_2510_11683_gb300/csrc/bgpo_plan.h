@@ -1,0 +1,146 @@
+// Workspace layout, tile geometry and work splitting shared by the host code
+// and the kernels of the BGPO LM-head ELBO path.
+#pragma once
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __CUDACC__
+#define BGPO_HD __host__ __device__ __forceinline__
+#else
+#define BGPO_HD inline
+#endif
+
+namespace bgpo {
+
+// ---- GEMM tile geometry (one CTA computes a 128 x 256 fp32 tile in TMEM) ----
+constexpr int kBM = 128;         // rows per tile = TMEM lanes
+constexpr int kBN = 256;         // columns per tile = TMEM columns per accumulator
+constexpr int kBK = 64;          // K per pipeline stage: one 128-byte swizzle row of bf16
+constexpr int kUmmaK = 16;       // K of one tcgen05.mma kind::f16 instruction
+constexpr int kStages = 4;       // TMA -> MMA pipeline depth
+constexpr int kMaxSplits = 16;   // split-K limit of the dX GEMM
+
+constexpr uint32_t kTileABytes = kBM * kBK * 2;   // 16 KB
+constexpr uint32_t kTileBBytes = kBN * kBK * 2;   // 32 KB
+constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
+constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /*barriers*/ + 1024 /*align*/;
+
+// ---- kernel ids (trace + device error "where") --------------------------------
+enum KernelId : int32_t {
+  KID_MASK_COMPACT = 0,
+  KID_GATHER = 1,
+  KID_LMHEAD_FWD = 2,
+  KID_LSE_COMBINE = 3,
+  KID_SEQ_REDUCE = 4,
+  KID_BOUND_COEFFS = 5,
+  KID_LMHEAD_DZ = 6,
+  KID_DX_GEMM = 7,
+  KID_DX_REDUCE = 8,
+  KID_DW_GEMM = 9,
+  KID_GROUP_ADV = 10,
+  KID_COUNT = 11
+};
+
+BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+BGPO_HD int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
+
+// Split-K count of the dX GEMM (K = vocabulary) for `mb` row blocks times
+// `tiles_n` column tiles on `num_sms` SMs: the smallest s whose wave-quantised
+// time ceil(tiles*s/sms)/s is within 8% of the ideal tiles/sms, else the best s.
+// s * mb never exceeds `row_block_cap`, which bounds the partial buffer
+// independently of the SM count.
+BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_sms, int64_t k_blocks,
+                      int64_t row_block_cap) {
+  const int64_t tiles_mn = mb * tiles_n;
+  if (tiles_mn <= 0 || num_sms <= 0) return 1;
+  int64_t smax = kMaxSplits;
+  if (k_blocks < smax) smax = k_blocks > 0 ? k_blocks : 1;
+  if (row_block_cap / mb < smax) smax = row_block_cap / mb > 0 ? row_block_cap / mb : 1;
+  const double ideal = (double)tiles_mn / (double)num_sms;
+  int best = 1;
+  double best_t = 1e300;
+  for (int s = 1; s <= smax; ++s) {
+    const double t = (double)ceil_div(tiles_mn * s, num_sms) / (double)s;
+    if (t <= ideal * 1.08) return s;
+    if (t < best_t) { best_t = t; best = s; }
+  }
+  return best;
+}
+
+// Geometry derived from the problem sizes (host and device agree on it).
+struct Geometry {
+  int64_t B, P, R, H, V;
+  int64_t m_cap;      // B * R: most masked rows a sample can have
+  int64_t m_pad;      // m_cap rounded up to a tile of rows
+  int64_t v_pad;      // V rounded up to 64 (row pitch of the dZ buffer)
+  int64_t n_vt;       // vocabulary tiles of kBN columns
+  int64_t tiles_h;    // hidden-size tiles of kBN columns
+  int64_t kb_v;       // K blocks of kBK over the vocabulary (dX GEMM)
+};
+
+BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64_t V) {
+  Geometry g;
+  g.B = B; g.P = P; g.R = R; g.H = H; g.V = V;
+  g.m_cap = B * R;
+  g.m_pad = round_up(g.m_cap, kBM);
+  g.v_pad = round_up(V, 64);
+  g.n_vt = ceil_div(V, kBN);
+  g.tiles_h = ceil_div(H, kBN);
+  g.kb_v = ceil_div(V, kBK);
+  return g;
+}
+
+// Device workspace layout. Every region starts on a 1024-byte boundary (TMA
+// tiles with 128-byte swizzle want 1024-byte aligned bases).
+struct WsLayout {
+  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M
+  size_t t;          // float[B]    t_{b,j}
+  size_t tnum;       // uint32[2B]  T numerator (t = T / D), (low, high) words
+  size_t seg_off;    // int32[B+1]  first compacted row of each sequence
+  size_t rows;       // int32[m_cap] b*R + i of each masked position, ascending
+  size_t tgt;        // int32[m_pad] target token of each compacted row
+  size_t tgt_logit;  // float[m_pad] z_{r, y_r}
+  size_t lse;        // float[m_pad] log-sum-exp of each row's logits
+  size_t logp;       // float[m_pad] log p(y_r)
+  size_t part;       // float2[m_pad * n_vt] (max, sum-exp) per (row, vocab tile)
+  size_t xm;         // bf16[m_pad * H] gathered masked hidden states
+  size_t dz;         // bf16[m_pad * v_pad] dL/dz of the current sample
+  size_t dxp;        // float[dxp_elems] split-K partials of dX
+  size_t dxp_elems;
+  size_t total;
+};
+
+BGPO_HD size_t align_ws(size_t x) { return (x + 1023) & ~(size_t)1023; }
+
+// Row blocks the split-K partial buffer holds: enough for every split choice.
+BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
+  const int64_t mb_max = g.m_pad / kBM;
+  return mb_max > kMaxSplits ? mb_max : kMaxSplits;
+}
+
+BGPO_HD WsLayout make_ws_layout(const Geometry& g) {
+  WsLayout L;
+  size_t o = 0;
+  L.err = o;       o = align_ws(o + 64);
+  L.t = o;         o = align_ws(o + 4 * (size_t)g.B);
+  L.tnum = o;      o = align_ws(o + 8 * (size_t)g.B);
+  L.seg_off = o;   o = align_ws(o + 4 * (size_t)(g.B + 1));
+  L.rows = o;      o = align_ws(o + 4 * (size_t)g.m_cap);
+  L.tgt = o;       o = align_ws(o + 4 * (size_t)g.m_pad);
+  L.tgt_logit = o; o = align_ws(o + 4 * (size_t)g.m_pad);
+  L.lse = o;       o = align_ws(o + 4 * (size_t)g.m_pad);
+  L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
+  L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
+  L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
+  L.dz = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.v_pad);
+  L.dxp_elems = (size_t)dxp_row_block_cap(g) * kBM * (size_t)g.H;
+  L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
+  L.total = o;
+  return L;
+}
+
+// Indices into the int32 error word.
+enum ErrField : int { ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3 };
+
+}  // namespace bgpo

@@ -1,0 +1,329 @@
+// Non-GEMM kernels of the BGPO LM-head ELBO path: the forward masking process
+// with row compaction, the gather of masked hidden states, the log-sum-exp
+// combine, the per-sequence ELBO reduction (Eq. 4), the bound coefficients
+// (Eq. 10, 13), the split-K reduction of dX and the group advantages (Eq. 18).
+#include <math.h>
+
+#include "bgpo_device.cuh"
+#include "bgpo_internal.h"
+#include "philox.cuh"
+
+namespace bgpo {
+
+namespace {
+
+constexpr int32_t kStatusInvalidArg = 1;   // BGPO_ERR_INVALID_ARG
+constexpr int32_t kStatusNonfinite = 5;    // BGPO_ERR_NONFINITE
+
+// Masked rows of the sample the workspace holds, or 0 (and an error) when the
+// workspace holds another sample than `j`.
+__device__ __forceinline__ int32_t rows_of_sample(int32_t* err, int32_t j, int32_t kid) {
+  const int32_t tag = err[ERR_SAMPLE];
+  if (tag != j) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) set_device_error(err, kStatusInvalidArg, kid * 16 + 1);
+    return 0;
+  }
+  return err[ERR_M];
+}
+
+// ---------------------------------------------------------------------------
+// Forward masking process (Sec. 2.1; Eq. 3, 5) + stable compaction.
+// One CTA of 1024 threads walks the (b, q) Philox blocks in ascending order,
+// 1024 blocks per round; a block-wide exclusive scan places every masked
+// position (b, i) at its rank, so rows[] is sorted by b * R + i.
+// ---------------------------------------------------------------------------
+constexpr int kScanThreads = 1024;
+
+__global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtrs w) {
+  __shared__ int32_t warp_excl[32];
+  __shared__ int32_t s_carry;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int64_t Q = ((int64_t)a.R + 3) / 4;
+  const int64_t nblk = (int64_t)a.B * Q;
+  const uint64_t d_over_2_24 = (a.t_mode == 1) ? (uint64_t)a.n_t : 1ull;   // D / 2^24
+  if (tid == 0) s_carry = 0;
+  __syncthreads();
+  for (int64_t base = 0; base < nblk; base += kScanThreads) {
+    const int64_t e = base + tid;
+    int32_t cnt = 0;
+    uint32_t bits = 0;
+    int32_t b = 0, q = 0;
+    if (e < nblk) {
+      b = (int32_t)(e / Q);
+      q = (int32_t)(e % Q);
+      const PhiloxOut ot = philox4x64_10(0, (uint64_t)b, (uint64_t)a.j, kStreamT, a.seed, 0);
+      const uint64_t u = ot.w[0] >> kU24Shift;
+      const uint64_t T = (a.t_mode == 1) ? ((uint64_t)a.j << 24) + u + 1 : u + 1;
+      const PhiloxOut om = philox4x64_10((uint64_t)q, (uint64_t)b, (uint64_t)a.j, kStreamMask, a.seed, 0);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int32_t i = 4 * q + k;
+        if (i < a.R) {
+          // u24 / 2^24 < T / D  <=>  u24 * (D / 2^24) < T   (exact integers)
+          const uint32_t bit = ((om.w[k] >> kU24Shift) * d_over_2_24 < T) ? 1u : 0u;
+          bits |= bit << k;
+          cnt += (int32_t)bit;
+          if (a.mask_out) a.mask_out[(int64_t)b * a.R + i] = (uint8_t)bit;
+        }
+      }
+      if (q == 0) {
+        const float tf = (float)((double)T / (double)(d_over_2_24 << 24));
+        w.t[b] = tf;
+        w.tnum[2 * b] = (uint32_t)T;
+        w.tnum[2 * b + 1] = (uint32_t)(T >> 32);
+        if (a.t_out) a.t_out[b] = tf;
+      }
+    }
+    // block-wide exclusive scan of cnt
+    int32_t incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    if (lane == 31) warp_excl[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+      const int32_t v = warp_excl[lane];
+      int32_t vi = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int32_t n = __shfl_up_sync(0xffffffffu, vi, o);
+        if (lane >= o) vi += n;
+      }
+      warp_excl[lane] = vi - v;
+    }
+    __syncthreads();
+    const int32_t excl = s_carry + warp_excl[wid] + incl - cnt;
+    if (e < nblk) {
+      if (q == 0) w.seg_off[b] = excl;
+      int32_t pos = excl;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if ((bits >> k) & 1u) w.rows[pos++] = b * a.R + 4 * q + k;
+    }
+    __syncthreads();
+    if (tid == kScanThreads - 1) s_carry = excl + cnt;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    const int32_t M = s_carry;
+    w.seg_off[a.B] = M;
+    w.err[ERR_M] = M;
+    w.err[ERR_SAMPLE] = a.j;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Gather of the masked rows' hidden states (the indicator of Eq. 4 selects
+// them): Xm[r] = X[b, P + i] with 16-byte vector copies, one warp per row.
+// Rows [M, round_up(M, 128)) are zero-filled so that the GEMM tiles and the
+// K padding of the dW GEMM read zeros.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_gather(Geometry g, int32_t j, const uint4* __restrict__ X,
+                                                const int32_t* __restrict__ Y, WsPtrs w) {
+  const int32_t M = rows_of_sample(w.err, j, KID_GATHER);
+  const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= round_up(M, kBM)) return;
+  const int64_t nvec = g.H / 8;
+  uint4* dst = reinterpret_cast<uint4*>(w.xm) + r * nvec;
+  if (r < M) {
+    const int32_t idx = w.rows[r];
+    const int64_t b = idx / g.R, i = idx % g.R;
+    const uint4* src = X + (b * (g.P + g.R) + g.P + i) * nvec;
+    for (int64_t v = lane; v < nvec; v += 32) dst[v] = __ldg(src + v);
+    if (lane == 0) w.tgt[r] = __ldg(Y + idx);
+  } else {
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    for (int64_t v = lane; v < nvec; v += 32) dst[v] = z;
+    if (lane == 0) w.tgt[r] = 0;
+  }
+}
+
+// (m, s) pairs represent s * e^m; merging keeps the larger exponent.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) { m = m2; s = s2; return; }
+  if (m2 > m) { s = s * expf(m - m2) + s2; m = m2; }
+  else        { s = s + s2 * expf(m2 - m); }
+}
+
+// ---------------------------------------------------------------------------
+// log-sum-exp of each masked row from the per-vocab-tile partials, then
+// log p(y_r) = z_{r, y_r} - lse_r. One warp per row, fixed merge order.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, WsPtrs w) {
+  const int32_t M = rows_of_sample(w.err, j, KID_LSE_COMBINE);
+  const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= M) return;
+  float m = -INFINITY, s = 0.f;
+  const float2* part = w.part + r * g.n_vt;
+  for (int64_t i = lane; i < g.n_vt; i += 32) {
+    const float2 p = part[i];
+    lse_merge(m, s, p.x, p.y);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    lse_merge(m, s, m2, s2);
+  }
+  if (lane == 0) {
+    const float lse = m + logf(s);
+    w.lse[r] = lse;
+    w.logp[r] = w.tgt_logit[r] - lse;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 4: l_b = (1/t_b) * sum over sequence b's masked rows of log p. One warp
+// per sequence, lane-strided sums then a fixed xor tree (deterministic).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_seq_reduce(Geometry g, int32_t j, WsPtrs w, float* ell_out) {
+  const int32_t M = rows_of_sample(w.err, j, KID_SEQ_REDUCE);
+  const int64_t b = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (b >= g.B) return;
+  float acc = 0.f;
+  if (M > 0) {
+    const int32_t lo = w.seg_off[b], hi = w.seg_off[b + 1];
+    for (int32_t r = lo + lane; r < hi; r += 32) acc += w.logp[r];
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) ell_out[b] = acc / w.t[b];
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 10 and 13 (Algorithm 1: L_j = -loss_scale * g_j):
+//   d = l - l_old; A >= 0: g = (1 + d) A / n_t, dg/dl = A / n_t (Lemma 1)
+//                  A <  0: g = e^d A / n_t,    dg/dl = e^d A / n_t (Lemma 2)
+// ---------------------------------------------------------------------------
+__global__ void k_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* __restrict__ ell,
+                               const float* __restrict__ ell_old, const float* __restrict__ A,
+                               float* coef_out, float* g_out, int32_t* err) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const float d = ell[b] - ell_old[b];
+  const float a = A[b];
+  const bool taylor = a >= 0.f;
+  const float kappa = taylor ? 1.f : expf(d);
+  const float inv_nt = 1.f / (float)n_t;
+  const float g = taylor ? (1.f + d) * a * inv_nt : kappa * a * inv_nt;
+  const float coef = -loss_scale * a * kappa * inv_nt;
+  coef_out[b] = coef;
+  if (g_out) g_out[b] = g;
+  if (!isfinite(g) || !isfinite(coef)) set_device_error(err, kStatusNonfinite, KID_BOUND_COEFFS * 16);
+}
+
+// ---------------------------------------------------------------------------
+// dX[b, i, :] += sum_s partial_s[r, :] over the split-K partials of the dX GEMM
+// (fixed split order; rows are unique within a sample, so no atomics).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, int num_sms, WsPtrs w,
+                                                   float* __restrict__ dX) {
+  const int32_t M = rows_of_sample(w.err, j, KID_DX_REDUCE);
+  const int64_t r = blockIdx.x;
+  if (r >= M) return;
+  const int64_t mb = ceil_div(M, kBM);
+  const int S = dx_splits(mb, g.tiles_h, num_sms, g.kb_v, dxp_row_block_cap(g));
+  const int64_t split_stride = mb * kBM * g.H / 4;
+  const float4* src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
+  float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)w.rows[r] * (g.H / 4);
+  for (int64_t h = threadIdx.x; h < g.H / 4; h += blockDim.x) {
+    float4 acc = src[h];
+    for (int s = 1; s < S; ++s) {
+      const float4 v = src[s * split_stride + h];
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
+    float4 o = dst[h];
+    o.x += acc.x; o.y += acc.y; o.z += acc.z; o.w += acc.w;
+    dst[h] = o;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 18 over consecutive groups of G rewards (population std; 0 if std = 0).
+// ---------------------------------------------------------------------------
+__global__ void k_group_advantage(int32_t B, int32_t G, const float* __restrict__ r, float* A) {
+  const int64_t grp = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (grp * G >= B) return;
+  const float* x = r + grp * G;
+  float mean = 0.f;
+  for (int k = 0; k < G; ++k) mean += x[k];
+  mean /= (float)G;
+  float var = 0.f;
+  for (int k = 0; k < G; ++k) var += (x[k] - mean) * (x[k] - mean);
+  const float sd = sqrtf(var / (float)G);
+  for (int k = 0; k < G; ++k) A[grp * G + k] = sd > 0.f ? (x[k] - mean) / sd : 0.f;
+}
+
+}  // namespace
+
+WsPtrs ws_pointers(void* ws, const WsLayout& L) {
+  char* base = static_cast<char*>(ws);
+  WsPtrs p;
+  p.err = reinterpret_cast<int32_t*>(base + L.err);
+  p.t = reinterpret_cast<float*>(base + L.t);
+  p.tnum = reinterpret_cast<uint32_t*>(base + L.tnum);
+  p.seg_off = reinterpret_cast<int32_t*>(base + L.seg_off);
+  p.rows = reinterpret_cast<int32_t*>(base + L.rows);
+  p.tgt = reinterpret_cast<int32_t*>(base + L.tgt);
+  p.tgt_logit = reinterpret_cast<float*>(base + L.tgt_logit);
+  p.lse = reinterpret_cast<float*>(base + L.lse);
+  p.logp = reinterpret_cast<float*>(base + L.logp);
+  p.part = reinterpret_cast<float2*>(base + L.part);
+  p.xm = base + L.xm;
+  p.dz = base + L.dz;
+  p.dxp = reinterpret_cast<float*>(base + L.dxp);
+  return p;
+}
+
+cudaError_t launch_mask_compact(const MaskArgs& a, const WsPtrs& w, cudaStream_t s) {
+  k_mask_compact<<<1, kScanThreads, 0, s>>>(a, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const Geometry& g, int32_t j, const void* X, const int32_t* Y,
+                          const WsPtrs& w, cudaStream_t s) {
+  const unsigned grid = (unsigned)ceil_div(g.m_pad, 8);
+  k_gather<<<grid, 256, 0, s>>>(g, j, static_cast<const uint4*>(X), Y, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lse_combine(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s) {
+  const unsigned grid = (unsigned)ceil_div(g.m_cap, 8);
+  k_lse_combine<<<grid, 256, 0, s>>>(g, j, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* ell_out,
+                              cudaStream_t s) {
+  const unsigned grid = (unsigned)ceil_div(g.B, 8);
+  k_seq_reduce<<<grid, 256, 0, s>>>(g, j, w, ell_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
+                                const float* ell_old, const float* A, float* coef_out,
+                                float* g_out, const WsPtrs& w, cudaStream_t s) {
+  k_bound_coeffs<<<(unsigned)ceil_div(B, 256), 256, 0, s>>>(B, n_t, loss_scale, ell, ell_old, A,
+                                                            coef_out, g_out, w.err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_sms, const WsPtrs& w, float* dX,
+                             cudaStream_t s) {
+  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, num_sms, w, dX);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
+                                   cudaStream_t s) {
+  const int64_t groups = B / G;
+  k_group_advantage<<<(unsigned)ceil_div(groups, 128), 128, 0, s>>>(B, G, rewards, A_out);
+  return cudaGetLastError();
+}
+
+}  // namespace bgpo

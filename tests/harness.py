@@ -1,0 +1,97 @@
+"""Test-side drivers: the BGPO inner loops (Algorithm 1) through the C ABI on the
+GPU, and the same loops through the fp64 oracle on the CPU, on the same seeded
+inputs."""
+import numpy as np
+
+from oracle import bgpo_oracle as O
+
+
+def ensure_built():
+    """Builds lib/libbgpo.so when it is missing (nvcc cross-compiles without a GPU)."""
+    import os
+    from paper_2510_11683_gb300 import build as B
+    if not os.path.exists(B.LIB_PATH):
+        B.build()
+    return B.LIB_PATH
+
+
+def to64(t):
+    """torch tensor (bf16/f32/int) -> numpy float64 / int64 (exact widening)."""
+    import torch
+    if t.dtype in (torch.int32, torch.int64):
+        return t.cpu().numpy().astype(np.int64)
+    return t.cpu().to(torch.float64).numpy()
+
+
+def oracle_advantages(wl, inp):
+    if inp["A"] is not None:
+        return to64(inp["A"])
+    return O.group_advantage(to64(inp["rewards"]), wl.G)
+
+
+def oracle_run(wl, inp, loss_scale=None):
+    """Algorithm 1 inner loops in fp64: draws, l_self, l_old = l_self + eps, bound, grads."""
+    X, W, Y = to64(inp["X"]), to64(inp["W"]), to64(inp["Y"])
+    ls = 1.0 / wl.G if loss_scale is None else loss_scale
+    A = oracle_advantages(wl, inp)
+    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode)
+    ell_self = O.elbo_all(X, W, Y, wl.P, ts, masks)
+    ell_old = ell_self + to64(inp["eps"])
+    out = O.bgpo_step(X, W, Y, wl.P, A, ell_old, ts, masks, ls)
+    out.update(ts=ts, masks=masks, A=A, ell_old=ell_old, ell_self=ell_self)
+    return out
+
+
+def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None):
+    """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
+
+    Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
+    masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
+    """
+    import torch
+    import paper_2510_11683_gb300 as bg
+
+    prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale)
+    ws = bg.alloc_workspace(prob, dev)
+    bg.clear_device_error(ws)
+    B, n_t = wl.B, wl.n_t
+    X, W, Y = inp["X"], inp["W"], inp["Y"]
+    if inp["A"] is not None:
+        A = inp["A"].contiguous()
+    else:
+        A = torch.empty(B, dtype=torch.float32, device=dev)
+        bg.group_advantage(prob, inp["rewards"], A)
+    t = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    masks = torch.empty((n_t, B, wl.R), dtype=torch.uint8, device=dev)
+    ell_self = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    for j in range(n_t):          # old-policy pass (same draws, Eq. 10)
+        bg.sample_mask(prob, j, ws, t[j], masks[j])
+        bg.elbo_fwd(prob, j, X, W, Y, ws, ell_self[j])
+    ell_old = (ell_self + inp["eps"].T.contiguous()).contiguous()
+    ell = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    coef = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    g = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    dX = torch.zeros((B, wl.R, wl.H), dtype=torch.float32, device=dev)
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+    for j in range(n_t):          # Algorithm 1, one MC sample at a time
+        bg.sample_mask(prob, j, ws)
+        bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+        bg.bound_coeffs(prob, j, ell[j], ell_old[j], A, coef[j], g[j], ws)
+        bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
+    torch.cuda.synchronize()
+    return dict(ell=ell.T, ell_old=ell_old.T, coef=coef.T, g=g.T, t=t, masks=masks, A=A,
+                dX=dX, dW=dW, ws=ws, prob=prob, ell_self=ell_self.T)
+
+
+def rel_ell_err(got, ref):
+    """|l_gpu - l_ref| / max(|l_ref|, 1) elementwise (the per-sequence tolerance rule)."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return np.abs(got - ref) / np.maximum(np.abs(ref), 1.0)
+
+
+def normwise(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    den = np.linalg.norm(ref)
+    return np.linalg.norm(got - ref) / (den if den > 0 else 1.0)

@@ -1,0 +1,170 @@
+"""C-ABI library: loads, exports every declared symbol, validates on the host.
+
+No GPU is needed: every call here either is host-only or fails validation
+before any CUDA call (on a machine without a GPU, a valid launching call
+returns BGPO_ERR_UNSUPPORTED_DEVICE instead of launching).
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from tests.harness import ensure_built
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    ensure_built()
+    from paper_2510_11683_gb300 import _lib
+    return _lib.lib()
+
+
+@pytest.fixture()
+def bg():
+    import paper_2510_11683_gb300 as bg
+    return bg
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "bgpo.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"\b(bgpo_[a-z_0-9]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(L):
+    from paper_2510_11683_gb300 import _lib
+    names = _declared_functions()
+    assert len(names) == len(_lib.SIGNATURES) == 17
+    for n in names:
+        assert hasattr(L, n), n
+        assert n in _lib.SIGNATURES, f"binding lacks {n}"
+
+
+def test_abi_version_and_names(L, bg):
+    assert L.bgpo_abi_version() == 1
+    assert L.bgpo_status_string(0) == b"BGPO_OK"
+    assert L.bgpo_status_string(8) == b"BGPO_ERR_TIMEOUT"
+    assert bg.kernel_name(2) == "lmhead_fwd_lse"
+    assert bg.kernel_name(99) == "?"
+
+
+def test_problem_struct_layout(bg):
+    assert ctypes.sizeof(bg.BgpoProblem) == 56
+    assert bg.BgpoProblem.seed.offset == 32
+    assert bg.BgpoProblem.trace.offset == 48
+
+
+def _prob(bg, **kw):
+    args = dict(B=2, P=16, R=32, H=64, V=512, n_t=4, G=2, t_mode=0, seed=1)
+    args.update(kw)
+    return bg.problem(**args)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(B=0), 2), (dict(R=0), 2), (dict(P=-1), 2), (dict(H=96), 2), (dict(H=0), 2),
+    (dict(V=0), 2), (dict(n_t=0), 2), (dict(n_t=65536), 2), (dict(G=0), 2),
+    (dict(t_mode=2), 1), (dict(B=1 << 12, R=1 << 11), 2), (dict(V=(1 << 24) + 1), 2),
+])
+def test_validation_rejects_bad_problems(L, bg, kw, status):
+    p = _prob(bg, **kw)
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == status
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
+
+
+def test_validation_rejects_flags_and_nonfinite_scale(L, bg):
+    p = _prob(bg)
+    p.flags = 1
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    p = _prob(bg, loss_scale=float("nan"))
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    assert L.bgpo_validate_problem(None) == 1
+
+
+def test_workspace_independent_of_n_t(L, bg):
+    sizes = {n: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, n_t=n))) for n in (1, 2, 16, 32, 1000)}
+    assert len(set(sizes.values())) == 1 and sizes[1] > 0
+
+
+def test_workspace_grows_with_rows_and_vocab(L, bg):
+    a = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg)))
+    assert L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=8))) > a
+    assert L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, V=4096))) > a
+
+
+def test_workspace_of_paper_shapes_fits_hbm(L, bg):
+    # LLaDA-8B head, 16 x 512 responses; Dream-7B head, 32 x 1024 (bytes, not n_t-dependent)
+    p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3)
+    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
+    p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5)
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 16e9
+
+
+FAKE = 1 << 20  # an aligned, never dereferenced address
+
+
+def test_sample_index_out_of_range(L, bg):
+    p = _prob(bg)
+    ws = L.bgpo_workspace_bytes(ctypes.byref(p))
+    for j in (-1, 4, 100):
+        assert L.bgpo_sample_mask(ctypes.byref(p), j, FAKE, ws, None, None, None) == 1
+        assert L.bgpo_elbo_fwd(ctypes.byref(p), j, FAKE, FAKE, FAKE, FAKE, ws, FAKE, None) == 1
+
+
+def test_null_and_misaligned_pointers(L, bg):
+    p = _prob(bg)
+    ws = L.bgpo_workspace_bytes(ctypes.byref(p))
+    assert L.bgpo_sample_mask(ctypes.byref(p), 0, None, ws, None, None, None) == 1
+    assert L.bgpo_sample_mask(ctypes.byref(p), 0, FAKE + 16, ws, None, None, None) == 3
+    assert L.bgpo_elbo_fwd(ctypes.byref(p), 0, None, FAKE, FAKE, FAKE, ws, FAKE, None) == 1
+    assert L.bgpo_elbo_fwd(ctypes.byref(p), 0, FAKE + 2, FAKE, FAKE, FAKE, ws, FAKE, None) == 3
+    assert L.bgpo_elbo_fwd(ctypes.byref(p), 0, FAKE, FAKE + 8, FAKE, FAKE, ws, FAKE, None) == 3
+    assert L.bgpo_bound_coeffs(ctypes.byref(p), 0, FAKE, None, FAKE, FAKE, None, FAKE, ws, None) == 1
+    assert L.bgpo_bound_coeffs(ctypes.byref(p), 0, FAKE + 1, FAKE, FAKE, FAKE, None, FAKE, ws, None) == 3
+    assert L.bgpo_elbo_bwd_accumulate(ctypes.byref(p), 0, FAKE, FAKE, FAKE, FAKE, FAKE, ws,
+                                      FAKE, None, None) == 1
+    assert L.bgpo_elbo_bwd_accumulate(ctypes.byref(p), 0, FAKE, FAKE, FAKE, FAKE, FAKE, ws,
+                                      FAKE + 4, FAKE, None) == 3
+    assert L.bgpo_group_advantage(ctypes.byref(p), None, FAKE, None) == 1
+
+
+def test_workspace_too_small(L, bg):
+    p = _prob(bg)
+    ws = L.bgpo_workspace_bytes(ctypes.byref(p))
+    assert L.bgpo_sample_mask(ctypes.byref(p), 0, FAKE, ws - 1, None, None, None) == 4
+    assert L.bgpo_elbo_bwd_accumulate(ctypes.byref(p), 0, FAKE, FAKE, FAKE, FAKE, FAKE, 1024,
+                                      FAKE, FAKE, None) == 4
+
+
+def test_group_size_must_divide_batch(L, bg):
+    p = _prob(bg, B=6, G=4)
+    assert L.bgpo_group_advantage(ctypes.byref(p), FAKE, FAKE, None) == 2
+
+
+def test_valid_call_without_gpu_reports_device(L, bg):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    p = _prob(bg)
+    ws = L.bgpo_workspace_bytes(ctypes.byref(p))
+    assert L.bgpo_sample_mask(ctypes.byref(p), 0, FAKE, ws, None, None, None) == 6
+
+
+def test_trace_api_without_events(L):
+    assert L.bgpo_trace_create(0) is None
+    assert L.bgpo_trace_count(None) == 0
+    L.bgpo_trace_reset(None)
+    L.bgpo_trace_destroy(None)
+    kid = ctypes.c_int32(0)
+    ms = ctypes.c_float(0)
+    assert L.bgpo_trace_get(None, 0, ctypes.byref(kid), ctypes.byref(ms)) == 1
+
+
+def test_binding_rejects_cpu_tensors(bg):
+    import torch
+    p = _prob(bg)
+    with pytest.raises(ValueError):
+        bg.sample_mask(p, 0, torch.zeros(16, dtype=torch.uint8))

@@ -1,0 +1,276 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Tolerances (spec contract): masks bit-exact; per-sequence l within 1e-3
+relative (|dl| <= 1e-3 max(|l|, 1)); accumulated dX, dW within 2e-2 normwise
+relative; bound coefficients within 1e-5 relative of the oracle on identical
+inputs (fp32 arithmetic of Eq. 10/13).
+"""
+import numpy as np
+import pytest
+
+from oracle import bgpo_oracle as O
+from synth import CONFIGS, make_inputs
+from tests.harness import ensure_built, gpu_run, normwise, oracle_run, rel_ell_err, to64
+
+pytestmark = pytest.mark.gpu
+
+ELL_TOL = 1e-3
+GRAD_TOL = 2e-2
+
+
+@pytest.fixture(scope="module")
+def bg():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    ensure_built()
+    import paper_2510_11683_gb300 as bg
+    return bg
+
+
+def _inputs(name, **over):
+    wl = CONFIGS[name].with_(**over) if over else CONFIGS[name]
+    return wl, make_inputs(wl, device="cuda")
+
+
+@pytest.fixture(scope="module")
+def runs(bg):
+    """GPU and oracle runs of the parity workloads (computed once per module)."""
+    out = {}
+    for name in ("tiny", "ragged", "ragged_strat"):
+        wl, inp = _inputs(name)
+        out[name] = (wl, inp, gpu_run(wl, inp), oracle_run(wl, {k: (v.cpu() if v is not None else None)
+                                                                 for k, v in inp.items()}))
+    return out
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged", "ragged_strat"])
+def test_masks_and_t_bit_exact(runs, name):
+    wl, inp, g, o = runs[name]
+    assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+    # t = T / D rounded once to float32 on both sides
+    assert np.array_equal(g["t"].cpu().numpy(), o["ts"].astype(np.float32))
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged", "ragged_strat"])
+def test_elbo_matches_oracle(runs, name):
+    wl, inp, g, o = runs[name]
+    err = rel_ell_err(to64(g["ell_self"]), o["ell_self"])
+    assert err.max() <= ELL_TOL, err.max()
+    err = rel_ell_err(to64(g["ell"]), o["ell"])
+    assert err.max() <= ELL_TOL, err.max()
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged", "ragged_strat"])
+def test_gradients_match_oracle(runs, name):
+    wl, inp, g, o = runs[name]
+    assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL
+    assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged", "ragged_strat"])
+def test_bound_values_match_oracle(runs, name):
+    wl, inp, g, o = runs[name]
+    # d is formed from each side's own l; with l_old = l_self + eps both give d = -eps
+    assert np.allclose(to64(g["g"]), o["g"], rtol=2e-3, atol=1e-5)
+    assert np.allclose(to64(g["coef"]), o["coef"], rtol=2e-3, atol=1e-6)
+
+
+def test_group_advantage_matches_oracle(bg):
+    import torch
+    rng = np.random.default_rng(5)
+    r = (rng.random(64) < 0.5).astype(np.float32)
+    r[:8] = 1.0   # a zero-std group
+    p = bg.problem(64, 1, 1, 64, 8, 1, 8)
+    A = torch.empty(64, dtype=torch.float32, device="cuda")
+    bg.group_advantage(p, torch.from_numpy(r).cuda(), A)
+    ref = O.group_advantage(r.astype(np.float64), 8)
+    assert np.allclose(A.cpu().numpy(), ref, rtol=1e-5, atol=1e-6)
+    assert np.array_equal(A[:8].cpu().numpy(), np.zeros(8, dtype=np.float32))
+
+
+def test_bound_coeffs_on_identical_inputs(bg):
+    import torch
+    rng = np.random.default_rng(7)
+    B, n_t = 300, 16
+    p = bg.problem(B, 1, 1, 64, 8, n_t, 8)
+    ws = bg.alloc_workspace(p)
+    bg.clear_device_error(ws)
+    bg.sample_mask(p, 3, ws)
+    ell = rng.standard_normal(B).astype(np.float32) * 50
+    ell_old = (ell + rng.standard_normal(B).astype(np.float32) * 0.5).astype(np.float32)
+    A = rng.standard_normal(B).astype(np.float32)
+    A[:5] = 0.0
+    cuda = lambda a: torch.from_numpy(a).cuda()
+    coef = torch.empty(B, device="cuda")
+    gg = torch.empty(B, device="cuda")
+    bg.bound_coeffs(p, 3, cuda(ell), cuda(ell_old), cuda(A), coef, gg, ws)
+    _, g_ref, c_ref = O.bound_coeffs(ell.astype(np.float64), ell_old.astype(np.float64),
+                                     A.astype(np.float64), n_t, 1.0 / 8)
+    assert np.allclose(coef.cpu().numpy(), c_ref, rtol=1e-5, atol=1e-9)
+    assert np.allclose(gg.cpu().numpy(), g_ref, rtol=1e-5, atol=1e-7)
+    assert bg.get_device_error(ws) == (0, 0)
+
+
+def test_backward_with_oracle_coefficients(bg):
+    """K6 isolated: oracle coefficients fed in, one sample, compared with the oracle."""
+    import torch
+    wl, inp = _inputs("ragged")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    bg.clear_device_error(ws)
+    rng = np.random.default_rng(3)
+    coef = rng.standard_normal(wl.B).astype(np.float64) * 0.3
+    ell = torch.empty(wl.B, device="cuda")
+    dX = torch.zeros((wl.B, wl.R, wl.H), device="cuda")
+    dW = torch.zeros((wl.V, wl.H), device="cuda")
+    j = 1
+    bg.sample_mask(p, j, ws)
+    bg.elbo_fwd(p, j, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_bwd_accumulate(p, j, inp["X"], inp["W"], inp["Y"],
+                           torch.from_numpy(coef.astype(np.float32)).cuda(), ws, dX, dW)
+    _, _, t, mask = O.sample_t_mask(wl.seed, wl.B, wl.R, j, wl.n_t, wl.t_mode)
+    gx, gw = O.elbo_term_grads(to64(inp["X"]), to64(inp["W"]), to64(inp["Y"]), wl.P, mask, t,
+                               coef.astype(np.float32).astype(np.float64))
+    assert normwise(to64(dW), gw) <= GRAD_TOL
+    assert normwise(to64(dX), gx) <= GRAD_TOL
+    assert bg.get_device_error(ws) == (0, 0)
+
+
+def test_forward_is_deterministic(bg):
+    import torch
+    wl, inp = _inputs("ragged")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    a = torch.empty(wl.B, device="cuda")
+    b = torch.empty(wl.B, device="cuda")
+    for out in (a, b):
+        bg.sample_mask(p, 2, ws)
+        bg.elbo_fwd(p, 2, inp["X"], inp["W"], inp["Y"], ws, out)
+    assert torch.equal(a, b)
+
+
+def test_on_policy_equivalence_on_gpu(bg):
+    """Sec. 3.2 on the device: d = 0 exactly, g n_t = A and coef = -A / (G n_t)."""
+    import torch
+    wl, inp = _inputs("ragged", eps_std=0.0)
+    g = gpu_run(wl, inp)
+    ell, ell_old = g["ell"].cpu().numpy(), g["ell_old"].cpu().numpy()
+    assert np.array_equal(ell, ell_old)
+    A = g["A"].cpu().numpy()
+    assert np.allclose(g["g"].cpu().numpy() * wl.n_t, A[:, None], rtol=1e-6, atol=1e-7)
+    assert np.allclose(g["coef"].cpu().numpy(), -A[:, None] / (wl.G * wl.n_t), rtol=1e-6, atol=1e-9)
+
+
+def test_dw_rows_sum_to_zero(runs):
+    """sum_v dz_{r,v} = 0 up to the bf16 rounding of dz: |sum_v dW| << |dW|."""
+    for name in ("tiny", "ragged"):
+        wl, inp, g, o = runs[name]
+        dW = to64(g["dW"])
+        col = np.abs(dW.sum(axis=0)).max()
+        assert col <= 1e-2 * np.abs(dW).sum(axis=0).max()
+
+
+def test_resume_at_sample_is_bit_identical(bg):
+    import torch
+    wl, inp = _inputs("tiny")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    full = []
+    for j in range(wl.n_t):
+        m = torch.empty((wl.B, wl.R), dtype=torch.uint8, device="cuda")
+        bg.sample_mask(p, j, ws, None, m)
+        full.append(m)
+    m2 = torch.empty((wl.B, wl.R), dtype=torch.uint8, device="cuda")
+    bg.sample_mask(p, 2, ws, None, m2)
+    assert torch.equal(full[2], m2)
+
+
+def test_empty_masks_give_zero(bg):
+    """R = 1 with small t: samples whose mask is empty give l = 0 and no gradient."""
+    import torch
+    wl = CONFIGS["tiny"].with_(B=1, R=1, n_t=64, P=3)
+    inp = make_inputs(wl, device="cuda")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    _, masks = O.sample_masks(wl.seed, 1, 1, wl.n_t, wl.t_mode)
+    empty_j = [j for j in range(wl.n_t) if masks[j].sum() == 0]
+    assert empty_j, "no empty sample drawn"
+    dX = torch.zeros((1, 1, wl.H), device="cuda")
+    dW = torch.zeros((wl.V, wl.H), device="cuda")
+    ell = torch.full((1,), 7.0, device="cuda")
+    coef = torch.ones(1, device="cuda")
+    j = empty_j[0]
+    bg.sample_mask(p, j, ws)
+    bg.elbo_fwd(p, j, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_bwd_accumulate(p, j, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    torch.cuda.synchronize()
+    assert float(ell[0]) == 0.0
+    assert float(dW.abs().max()) == 0.0 and float(dX.abs().max()) == 0.0
+
+
+def test_all_rows_masked(bg):
+    """Stratified t close to 1 masks (nearly) every row: M = B * R edge."""
+    import torch
+    wl = CONFIGS["ragged"].with_(t_mode=1, n_t=64, R=40)
+    inp = make_inputs(wl, device="cuda")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    j = 63
+    _, _, t, mask = O.sample_t_mask(wl.seed, wl.B, wl.R, j, wl.n_t, wl.t_mode)
+    ell = torch.empty(wl.B, device="cuda")
+    bg.sample_mask(p, j, ws)
+    bg.elbo_fwd(p, j, inp["X"], inp["W"], inp["Y"], ws, ell)
+    ref = O.elbo_term(to64(inp["X"]), to64(inp["W"]), to64(inp["Y"]), wl.P, mask, t)
+    assert mask.mean() > 0.9
+    assert rel_ell_err(ell.cpu().numpy(), ref).max() <= ELL_TOL
+
+
+def test_stale_sample_sets_device_error(bg):
+    import torch
+    wl, inp = _inputs("tiny")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    bg.clear_device_error(ws)
+    bg.sample_mask(p, 0, ws)
+    ell = torch.empty(wl.B, device="cuda")
+    bg.elbo_fwd(p, 1, inp["X"], inp["W"], inp["Y"], ws, ell)   # workspace holds sample 0
+    code, where = bg.get_device_error(ws)
+    assert code == 1
+    assert float(ell.abs().max()) == 0.0
+    bg.clear_device_error(ws)
+    assert bg.get_device_error(ws) == (0, 0)
+
+
+def test_nonfinite_coefficient_sets_device_error(bg):
+    import torch
+    p = bg.problem(4, 1, 1, 64, 8, 2, 2)
+    ws = bg.alloc_workspace(p)
+    bg.clear_device_error(ws)
+    ell = torch.tensor([1.0, 2.0, 500.0, 0.0], device="cuda")
+    old = torch.zeros(4, device="cuda")
+    A = torch.tensor([1.0, -1.0, -1.0, 1.0], device="cuda")   # e^500 overflows fp32
+    coef = torch.empty(4, device="cuda")
+    bg.bound_coeffs(p, 0, ell, old, A, coef, None, ws)
+    assert bg.get_device_error(ws)[0] == 5
+
+
+def test_trace_records_every_kernel(bg):
+    import torch
+    wl, inp = _inputs("tiny")
+    tr = bg.Trace(64)
+    p = bg.problem_from(wl, trace=tr)
+    ws = bg.alloc_workspace(p)
+    ell = torch.empty(wl.B, device="cuda")
+    coef = torch.zeros(wl.B, device="cuda")
+    dX = torch.zeros((wl.B, wl.R, wl.H), device="cuda")
+    dW = torch.zeros((wl.V, wl.H), device="cuda")
+    bg.sample_mask(p, 0, ws)
+    bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.bound_coeffs(p, 0, ell, ell, inp["A"], coef, None, ws)
+    bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    names = [n for n, ms in tr.records()]
+    assert names == ["mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
+                     "bound_coeffs", "lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
+    assert all(ms >= 0 for _, ms in tr.records())
+    tr.close()
