@@ -1,0 +1,475 @@
+"""Throughput of the BGPO masked-diffusion ELBO hot path on GB300.
+
+One step = Algorithm 1's inner loops over one batch: for every MC sample j,
+sample_mask -> elbo_fwd -> bound_coeffs -> elbo_bwd_accumulate, through the C ABI
+of include/bgpo.h (all arithmetic in the library's CUDA kernels). Workload:
+LLaDA-8B-shaped LM head (H=4096, V=126464), 16 responses of 512 tokens after a
+256-token prompt, n_t=16 stratified MC samples, on-policy (old = current).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints ONE JSON line (rank 0). `value` = masked tokens/s over all ranks with
+inputs resident in HBM; `e2e` = the same through host (pinned) buffers with the
+host<->device copies inside the timed region; `roofline` = the dominant kernel's
+algorithmic tensor FLOP/s against the measured bf16 peak; `cpu_baseline` = the
+fp64 oracle on a bounded sample of the same workload on the host cores.
+`--impl reference` times that oracle alone (the reference arm of this tier).
+"""
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "llada8b_r512_onpolicy"
+METRIC = "masked tokens/s (fwd+bwd)"
+UNIT = "tokens/s"
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant kernel,
+# from the ncu capture summarised in profiles/ (scaled to this workload's masked
+# rows per launch). Valid only while the kernel source is unchanged.
+TRAFFIC = {
+    # kernel name: (bytes per masked row, sha256 of k_gemm.cu when captured)
+}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return dict(bf16=float(d["bf16_tflops"]), bf16_sustained=float(d["bf16_tflops_sustained"]),
+                    hbm=float(d["hbm_gbs"]), source="measured")
+    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(smax),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------------
+# CPU baseline / reference arm: the fp64 oracle as it stands, on a bounded sample
+# ----------------------------------------------------------------------------------
+
+def oracle_sample(wl, inp_cpu, budget_s=12.0, max_seqs=4):
+    """Times the oracle's per-sample path (Eq. 4 forward, Eq. 10/13 bound, gradients)
+    for MC sample j = n_t/2 on sequences 0, 1, ... until `budget_s` has passed.
+    Returns (masked rows processed, seconds, description)."""
+    from oracle import bgpo_oracle as O
+    from tests.harness import to64
+
+    X = to64(inp_cpu["X"])
+    W = to64(inp_cpu["W"])
+    Y = to64(inp_cpu["Y"])
+    j = wl.n_t // 2
+    _, _, t, mask = O.sample_t_mask(wl.seed, wl.B, wl.R, j, wl.n_t, wl.t_mode)
+    rows = 0
+    seqs = 0
+    t0 = time.perf_counter()
+    for b in range(min(wl.B, max_seqs)):
+        sub = np.zeros_like(mask)
+        sub[b] = mask[b]
+        ell = O.elbo_term(X, W, Y, wl.P, sub, t)
+        _, _, coef = O.bound_coeffs(ell, ell, np.ones(wl.B), wl.n_t, 1.0 / wl.G)
+        O.elbo_term_grads(X, W, Y, wl.P, sub, t, coef)
+        rows += int(mask[b].sum())
+        seqs += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    desc = (f"oracle fp64 (numpy, BLAS on all host cores): MC sample j={j} of sequences "
+            f"0..{seqs - 1} ({rows} masked rows, full V={wl.V}, H={wl.H}): forward, bound "
+            f"coefficients and gradients")
+    return rows, dt, desc
+
+
+def run_reference(args, wl):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from synth import make_inputs
+    inp = make_inputs(wl)
+    for _ in range(args.warmup):
+        oracle_sample(wl, inp, budget_s=2.0, max_seqs=1)
+    tot_rows, tot_s = 0, 0.0
+    desc = ""
+    for _ in range(args.steps):
+        rows, dt, desc = oracle_sample(wl, inp, budget_s=4.0, max_seqs=1)
+        tot_rows += rows
+        tot_s += dt
+    value = tot_rows / tot_s
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(wl),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_of(wl):
+    return {"workload": f"{wl.name}: LLaDA-8B-shaped LM head H={wl.H} V={wl.V}, {wl.B} responses "
+                        f"x (prompt {wl.P} + response {wl.R}), n_t={wl.n_t} "
+                        f"{'stratified' if wl.t_mode else 'iid'} t, G={wl.G}, "
+                        f"{'on-policy' if wl.eps_std == 0 else 'off-policy'}",
+            "B": wl.B, "P": wl.P, "R": wl.R, "H": wl.H, "V": wl.V, "n_t": wl.n_t, "G": wl.G,
+            "l2": "inputs larger than L2 (W alone is 1.04 GB > 129 MB); no flush"}
+
+
+# ----------------------------------------------------------------------------------
+# native arm
+# ----------------------------------------------------------------------------------
+
+def kernel_sha():
+    with open(os.path.join(ROOT, "paper_2510_11683_gb300", "csrc", "k_gemm.cu"), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def main():
+    args = parse()
+    from synth import CONFIGS
+    wl = CONFIGS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+        return
+
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2510_11683_gb300 as bg
+    from paper_2510_11683_gb300 import build as B
+    if not os.path.exists(B.LIB_PATH):
+        B.build()
+    from synth import make_inputs
+
+    # weak scaling: every rank owns its own batch of responses (independent units)
+    wl_r = wl.with_(seed=wl.seed + 1000 * rank) if world > 1 else wl
+    inp_cpu = make_inputs(wl_r)
+    inp = {k: (v.to(dev) if v is not None else None) for k, v in inp_cpu.items()}
+    X, W, Y = inp["X"], inp["W"], inp["Y"]
+    n_t, Bsz = wl.n_t, wl.B
+
+    prob = bg.problem_from(wl_r)
+    ws = bg.alloc_workspace(prob, dev)
+    bg.clear_device_error(ws)
+    A = torch.empty(Bsz, dtype=torch.float32, device=dev)
+    if inp["A"] is not None:
+        A.copy_(inp["A"])
+    else:
+        bg.group_advantage(prob, inp["rewards"], A)
+
+    # old-policy pass (outside the timed step): l_old on the same draws (Eq. 10)
+    ell_old = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
+    masks = torch.empty((n_t, Bsz, wl.R), dtype=torch.uint8, device=dev)
+    for j in range(n_t):
+        bg.sample_mask(prob, j, ws, None, masks[j])
+        bg.elbo_fwd(prob, j, X, W, Y, ws, ell_old[j])
+    ell_old += inp["eps"].T.to(dev)
+    masked_per_step = int(masks.sum().item())
+    rows_per_sample = masks.reshape(n_t, -1).sum(dim=1).tolist()
+
+    ell = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
+    coef = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
+    g = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
+    dX = torch.zeros((Bsz, wl.R, wl.H), dtype=torch.float32, device=dev)
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+
+    def step(p, X_, W_, Y_, A_, old_):
+        for j in range(n_t):
+            bg.sample_mask(p, j, ws)
+            bg.elbo_fwd(p, j, X_, W_, Y_, ws, ell[j])
+            bg.bound_coeffs(p, j, ell[j], old_[j], A_, coef[j], g[j], ws)
+            bg.elbo_bwd_accumulate(p, j, X_, W_, Y_, coef[j], ws, dX, dW)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step(prob, X, W, Y, A, ell_old)
+    torch.cuda.synchronize()
+
+    trace = bg.Trace(args.steps * n_t * 12 + 16)
+    prob_t = bg.problem_from(wl_r, trace=trace)
+    clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+    stream = torch.cuda.current_stream()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step(prob_t, X, W, Y, A, ell_old)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clock_info = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    code, where = bg.get_device_error(ws)
+    if code != 0:
+        raise RuntimeError(f"device error {code} at {where}")
+
+    recs = trace.records()
+    gpu_launches = len(recs)
+    per_kernel = {}
+    for name, kms in recs:
+        d = per_kernel.setdefault(name, [0, 0.0])
+        d[0] += 1
+        d[1] += kms
+    trace.close()
+
+    peaks = load_peaks()
+    H, V = wl.H, wl.V
+    gemm_flops_per_step = 2.0 * H * V * masked_per_step   # each of the four GEMMs
+    gemm_kernels = ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
+    dom = max(gemm_kernels, key=lambda k: per_kernel.get(k, [0, 0.0])[1])
+    dom_launches, dom_ms = per_kernel[dom]
+    dom_flops_per_launch = gemm_flops_per_step * args.steps / dom_launches
+    dom_avg_s = dom_ms / dom_launches / 1e3
+    achieved = dom_flops_per_launch / dom_avg_s / 1e12
+    traffic = None
+    if dom in TRAFFIC and TRAFFIC[dom][1] == kernel_sha():
+        traffic = TRAFFIC[dom][0] * masked_per_step / n_t
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
+                "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
+                "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
+                "flops_per_launch": dom_flops_per_launch, "avg_launch_ms": dom_avg_s * 1e3}
+
+    value = masked_per_step * world / (ms / 1e3)
+    exec_tflops = 4 * gemm_flops_per_step / (ms / 1e3) / 1e12
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; shapes of the paper's "
+        "LLaDA-8B head, response 512, n_t=16)", "config": config_of(wl),
+        "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clock_info,
+        "mc_samples_per_s": Bsz * n_t * world / (ms / 1e3),
+        "masked_rows_per_step": masked_per_step, "masked_rows_per_sample": rows_per_sample,
+        "step_tensor_tflops_executed": exec_tflops,
+        "step_frac_of_bf16_peak_executed": exec_tflops / peaks["bf16"],
+        "step_frac_of_bf16_peak_useful": 0.75 * exec_tflops / peaks["bf16"],
+        "per_kernel_ms_per_step": {k: v[1] / args.steps for k, v in per_kernel.items()},
+        "peak_mem_bytes": torch.cuda.max_memory_allocated(dev),
+        "workspace_bytes": ws.numel(),
+    }
+
+    if rank == 0 and world == 1 and not args.no_e2e:
+        out["e2e"] = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev)
+    elif rank == 0 and world > 1:
+        out["e2e"] = None
+
+    if rank == 0 and world == 1 and not args.no_sweep:
+        del dX, dW
+        torch.cuda.empty_cache()
+        out["nt_sweep"] = nt_sweep(bg, dev)
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rows, dt, desc = oracle_sample(wl, inp_cpu)
+        out["cpu_baseline"] = {"value": rows / dt, "unit": UNIT, "cores": os.cpu_count(),
+                               "kind": "oracle", "sample": desc, "seconds": dt}
+
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev):
+    """Same step through host buffers: pinned H2D of X, W, Y, A (or rewards) and
+    l_old, the n_t-sample loop, D2H of l and g; copies inside the timed region."""
+    import torch
+    n_t, Bsz = wl.n_t, wl.B
+    host = {
+        "X": inp_cpu["X"].pin_memory(), "W": inp_cpu["W"].pin_memory(),
+        "Y": inp_cpu["Y"].pin_memory(), "old": ell_old_cpu.contiguous().pin_memory(),
+    }
+    adv_key = "A" if inp_cpu["A"] is not None else "rewards"
+    host["adv"] = inp_cpu[adv_key].pin_memory()
+    dev_b = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+    out_ell = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
+    out_g = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
+    prob = bg.problem_from(wl)
+    ws = bg.alloc_workspace(prob, dev)
+    A = torch.empty(Bsz, dtype=torch.float32, device=dev)
+    ell = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
+    coef = torch.empty_like(ell)
+    g = torch.empty_like(ell)
+    dX = torch.zeros((Bsz, wl.R, wl.H), dtype=torch.float32, device=dev)
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = out_ell.numel() * 4 + out_g.numel() * 4
+
+    def step():
+        for k in host:
+            dev_b[k].copy_(host[k], non_blocking=True)
+        if adv_key == "A":
+            A.copy_(dev_b["adv"])
+        else:
+            bg.group_advantage(prob, dev_b["adv"], A)
+        for j in range(n_t):
+            bg.sample_mask(prob, j, ws)
+            bg.elbo_fwd(prob, j, dev_b["X"], dev_b["W"], dev_b["Y"], ws, ell[j])
+            bg.bound_coeffs(prob, j, ell[j], dev_b["old"][j], A, coef[j], g[j], ws)
+            bg.elbo_bwd_accumulate(prob, j, dev_b["X"], dev_b["W"], dev_b["Y"], coef[j], ws, dX, dW)
+        out_ell.copy_(ell, non_blocking=True)
+        out_g.copy_(g, non_blocking=True)
+
+    for _ in range(max(1, min(args.warmup, 2))):
+        step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, 5))
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+        torch.cuda.synchronize()       # the result is read on the host every step
+    dt = (time.perf_counter() - t0) / steps
+    return {"value": masked_per_step / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps}
+
+
+def nt_sweep(bg, dev):
+    """Time and peak memory of one step vs n_t (8 x (256 + 512), LLaDA-8B head)."""
+    import torch
+    from synth import CONFIGS, SWEEP_NT, make_inputs
+    base = CONFIGS["llada8b_sweep"]
+    inp0 = make_inputs(base.with_(n_t=max(SWEEP_NT)))
+    res = []
+    for n_t in SWEEP_NT:
+        wl = base.with_(n_t=n_t)
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats(dev)
+        X, W, Y = inp0["X"].to(dev), inp0["W"].to(dev), inp0["Y"].to(dev)
+        prob = bg.problem_from(wl)
+        ws = bg.alloc_workspace(prob, dev)
+        A = torch.empty(wl.B, dtype=torch.float32, device=dev)
+        bg.group_advantage(prob, inp0["rewards"].to(dev), A)
+        ell = torch.empty((n_t, wl.B), dtype=torch.float32, device=dev)
+        coef, g = torch.empty_like(ell), torch.empty_like(ell)
+        dX = torch.zeros((wl.B, wl.R, wl.H), dtype=torch.float32, device=dev)
+        dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+        rows = 0
+
+        def run():
+            for j in range(n_t):
+                bg.sample_mask(prob, j, ws)
+                bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+                bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
+                bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
+        run()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        run()
+        e1.record()
+        torch.cuda.synchronize()
+        m = torch.empty((wl.B, wl.R), dtype=torch.uint8, device=dev)
+        for j in range(n_t):
+            bg.sample_mask(prob, j, ws, None, m)
+            rows += int(m.sum().item())
+        res.append({"n_t": n_t, "ms": e0.elapsed_time(e1), "masked_rows": rows,
+                    "tokens_per_s": rows / (e0.elapsed_time(e1) / 1e3),
+                    "peak_bytes": torch.cuda.max_memory_allocated(dev)})
+        del X, W, Y, ws, dX, dW
+    return res
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,112 @@
+"""GPU parity at the paper-shaped sizes (full LM heads, full batches, all n_t).
+
+The whole Algorithm-1 loop runs exactly as bench.py runs it. The oracle checks
+what it can compute one by one at these sizes: every mask bit, the per-sequence
+l of the cheapest MC sample, the bound coefficients (the old-policy
+perturbation fixes d = -eps on both sides), sampled rows of dX; and properties
+that hold at any size: sum_v dW[v, :] ~ 0, on-policy d = 0 exactly, a clean
+device error word. Complete dW parity at the full head is checked with few
+masked rows.
+"""
+import numpy as np
+import pytest
+
+from oracle import bgpo_oracle as O
+from synth import CONFIGS, make_inputs
+from tests.harness import ensure_built, gpu_run, normwise, oracle_advantages, rel_ell_err, to64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def bg():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    ensure_built()
+    import paper_2510_11683_gb300 as bg
+    return bg
+
+
+def _sampled_dx_rows(wl, X, W, Y, ts, masks, coef, picks):
+    """Oracle dX[b, i] for a few response positions: sum over the samples that mask them."""
+    out = []
+    for b, i in picks:
+        x = X[b, wl.P + i]
+        z = W @ x
+        m = z.max()
+        p = np.exp(z - m)
+        p /= p.sum()
+        dz = -p
+        dz[int(Y[b, i])] += 1.0
+        wsum = sum(coef[b, j] / ts[j, b] for j in range(wl.n_t) if masks[j, b, i])
+        out.append(wsum * (W.T @ dz))
+    return np.stack(out)
+
+
+@pytest.mark.parametrize("name", ["llada8b_r256", "llada8b_r512_onpolicy", "dream7b"])
+def test_full_size_workload(bg, name):
+    import torch
+    wl = CONFIGS[name]
+    inp_cpu = make_inputs(wl)
+    inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
+    g = gpu_run(wl, inp)
+    assert bg.get_device_error(g["ws"]) == (0, 0)
+
+    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode)
+    assert np.array_equal(g["masks"].cpu().numpy(), masks)
+    assert np.array_equal(g["t"].cpu().numpy(), ts.astype(np.float32))
+
+    X, Y = to64(inp_cpu["X"]), to64(inp_cpu["Y"])
+    W = to64(inp_cpu["W"])
+    # per-sequence l of the 8 (sequence, sample) pairs with the fewest masked rows
+    counts = masks.sum(axis=2)                      # [n_t, B]
+    order = np.argsort(np.where(counts > 0, counts, 1 << 30), axis=None)[:8]
+    ell_gpu = to64(g["ell"])                        # [B, n_t]
+    for flat in order:
+        j, b = np.unravel_index(flat, counts.shape)
+        sub = np.zeros_like(masks[j])
+        sub[b] = masks[j, b]
+        ref = O.elbo_term(X, W, Y, wl.P, sub, ts[j])[b]
+        assert rel_ell_err([ell_gpu[b, j]], [ref]).max() <= 1e-3, (b, j)
+
+    # bound coefficients: l_old = l_self + eps gives d = -eps on both sides
+    A = oracle_advantages(wl, inp_cpu)
+    eps = to64(inp_cpu["eps"])
+    zero = np.zeros_like(eps)
+    _, g_ref, coef_ref = O.bound_coeffs(zero, zero + eps, A[:, None], wl.n_t, 1.0 / wl.G)
+    coef = to64(g["coef"])
+    assert np.allclose(coef, coef_ref, rtol=1e-4, atol=1e-9)
+    if wl.eps_std == 0.0:   # Equivalence (Sec. 3.2) on the device: d = 0 exactly
+        assert torch.equal(g["ell"], g["ell_old"])
+        assert np.allclose(to64(g["g"]) * wl.n_t, A[:, None], rtol=1e-5, atol=1e-6)
+
+    # sampled dX rows (positions masked at least once)
+    rng = np.random.default_rng(0)
+    hit = np.argwhere(masks.any(axis=0))
+    picks = [tuple(hit[k]) for k in rng.choice(len(hit), size=6, replace=False)]
+    ref = _sampled_dx_rows(wl, X, W, Y, ts, masks, coef_ref, picks)
+    got = np.stack([to64(g["dX"][b, i]) for b, i in picks])
+    assert normwise(got, ref) <= 2e-2
+
+    # sum_v dz_{r, v} = 0 up to the bf16 rounding of dz
+    dW = g["dW"]
+    colsum = dW.double().sum(dim=0).abs().max().item()
+    scale = dW.double().abs().sum(dim=0).max().item()
+    assert colsum <= 1e-2 * scale
+    assert torch.isfinite(dW).all() and torch.isfinite(g["dX"]).all()
+
+
+def test_full_head_complete_dw_parity(bg):
+    """Full LLaDA-8B head (494 vocabulary tiles, K = 4096) with few masked rows:
+    the whole dW and dX against the oracle."""
+    from tests.harness import oracle_run
+    wl = CONFIGS["llada8b_r256"].with_(B=2, P=8, R=24, n_t=2, G=2)
+    inp_cpu = make_inputs(wl)
+    inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
+    g = gpu_run(wl, inp)
+    o = oracle_run(wl, inp_cpu)
+    assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+    assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= 1e-3
+    assert normwise(to64(g["dW"]), o["dW"]) <= 2e-2
+    assert normwise(to64(g["dX"]), o["dX"]) <= 2e-2
