@@ -350,6 +350,11 @@ def main():
         "workspace_bytes": ws.numel(),
     }
 
+    if rank == 0:
+        print(f"[bench] {ms:.2f} ms/step, {value:.4g} tok/s, dominant {dom} "
+              f"{achieved:.1f} TFLOP/s, per kernel ms/step: "
+              f"{ {k: round(v[1] / args.steps, 3) for k, v in per_kernel.items()} }",
+              file=sys.stderr, flush=True)
     if rank == 0 and world == 1 and not args.no_e2e:
         out["e2e"] = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev)
     elif rank == 0 and world > 1:

@@ -76,7 +76,9 @@ def test_full_size_workload(bg, name):
     zero = np.zeros_like(eps)
     _, g_ref, coef_ref = O.bound_coeffs(zero, zero + eps, A[:, None], wl.n_t, 1.0 / wl.G)
     coef = to64(g["coef"])
-    assert np.allclose(coef, coef_ref, rtol=1e-4, atol=1e-9)
+    # l_old = l_self + eps is formed in fp32 on the device: at |l| up to ~2e4 its
+    # rounding moves d by up to ~1e-3, and the Jensen weight e^d with it
+    assert np.allclose(coef, coef_ref, rtol=2e-3, atol=1e-9)
     if wl.eps_std == 0.0:   # Equivalence (Sec. 3.2) on the device: d = 0 exactly
         assert torch.equal(g["ell"], g["ell_old"])
         assert np.allclose(to64(g["g"]) * wl.n_t, A[:, None], rtol=1e-5, atol=1e-6)
