@@ -61,6 +61,10 @@ CONFIGS = {
                                       V=126464, n_t=16, G=8, t_mode=1, seed=3,
                                       targets="zipf", zipf_s=1.1, advantages="bernoulli",
                                       eps_std=0.0),
+    # half of the batch above: the small case for full ncu captures (~4.5 GB on device)
+    "llada8b_r512_b8": Workload("llada8b_r512_b8", B=8, P=256, R=512, H=4096, V=126464, n_t=16,
+                                G=8, t_mode=1, seed=6, targets="zipf", zipf_s=1.1,
+                                advantages="bernoulli", eps_std=0.0),
     # n_t sweep (n_t overridden per point)
     "llada8b_sweep": Workload("llada8b_sweep", B=8, P=256, R=512, H=4096, V=126464, n_t=1, G=8,
                               t_mode=0, seed=4, targets="zipf", zipf_s=1.1,
