@@ -201,6 +201,34 @@ bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards,
                                  void* stream);
 
 /*
+ * bgpo_elbo_fwd_noalloc -- bgpo_sample_mask(j) followed by bgpo_elbo_fwd(j)
+ * with no caller-provided workspace: the scratch lives in a fixed array
+ * compiled into the library. The paper has no counterpart; this entry point
+ * exists for callers that cannot allocate device memory -- host code given
+ * only its input and output buffers by a process that plans all device
+ * memory itself, or code that must not call cudaMalloc because it would
+ * synchronise the device -- and so cannot pass the workspace the other calls
+ * need.
+ *   X, W, Y   as for bgpo_elbo_fwd;  t_out device float [B] or NULL;
+ *   ell_out   device float [B]: l_{b,j} (Eq. 4), same values as bgpo_elbo_fwd.
+ * Limit: the forward scratch of `prob` must fit the 32 MiB array, about
+ * roundup(B*R, 128) * (2 H + 8 ceil(V / 256) + 20) bytes; larger problems
+ * return BGPO_ERR_WORKSPACE_TOO_SMALL before anything is launched.
+ * Every GPU that loads the library holds the 32 MiB until the process exits.
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); that first call should
+ * come before any stream capture. Calls allocate nothing and free nothing.
+ * All calls share the one array, which keeps the previous call's contents:
+ * calls whose GPU work overlaps (other streams, other host threads) race and
+ * give undefined results. Device-side errors are recorded in the array's own
+ * error word, which the next call clears; use bgpo_elbo_fwd with a workspace
+ * to read them.
+ */
+bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j, const void* X,
+                                  const void* W, const int32_t* Y, float* t_out, float* ell_out,
+                                  void* stream);
+
+/*
  * Reads the device error word of a workspace (synchronises `stream`).
  *   code_out: BGPO_OK or the first device-detected status; where_out (may be
  *   NULL): kernel and site that set it.

@@ -42,6 +42,8 @@ SIGNATURES = {
                                            c_void_p, c_void_p, c_void_p, c_size_t, c_void_p,
                                            c_void_p, c_void_p]),
     "bgpo_group_advantage": (c_int32, [ctypes.POINTER(BgpoProblem), c_void_p, c_void_p, c_void_p]),
+    "bgpo_elbo_fwd_noalloc": (c_int32, [ctypes.POINTER(BgpoProblem), c_int32, c_void_p, c_void_p,
+                                        c_void_p, c_void_p, c_void_p, c_void_p]),
     "bgpo_get_device_error": (c_int32, [c_void_p, c_size_t, ctypes.POINTER(c_int32),
                                         ctypes.POINTER(c_int32), c_void_p]),
     "bgpo_clear_device_error": (c_int32, [c_void_p, c_size_t, c_void_p]),

@@ -19,7 +19,7 @@ OBJ_DIR = os.path.join(PKG_DIR, "_build")
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
                 f"-I{INCLUDE}", f"-I{CSRC}"]
-SOURCES = ["k_gemm.cu", "k_small.cu", "bgpo_api.cu"]
+SOURCES = ["k_gemm.cu", "k_small.cu", "bgpo_api.cu", "bgpo_noalloc.cu"]
 
 
 def nvcc():
