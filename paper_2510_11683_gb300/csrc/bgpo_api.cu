@@ -116,18 +116,20 @@ EncodeTiledFn encode_tiled() {
   return fn;
 }
 
-// 2-D bf16 tensor map over a row-major [outer, inner] matrix with row pitch
-// `pitch_bytes`, 128-byte swizzle, zero fill outside the matrix.
+// 2-D tensor map over a row-major [outer, inner] matrix with row pitch
+// `pitch_bytes`, 128-byte swizzle, zero fill outside the matrix (bf16 by
+// default, fp32 for the fp32 epilogue destinations).
 bool map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
-            uint32_t box_inner, uint32_t box_outer) {
+            uint32_t box_inner, uint32_t box_outer,
+            CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   EncodeTiledFn enc = encode_tiled();
   if (!enc) return false;
   const cuuint64_t dims[2] = {inner, outer};
   const cuuint64_t strides[1] = {pitch_bytes};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  return enc(m, dtype, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -205,11 +207,11 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
 
   CUtensorMap map_xm, map_w;
   if (!map_2d(&map_xm, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
-      !map_2d(&map_w, W, g.H, g.V, g.H * 2, kBK, kBN))
+      !map_2d(&map_w, W, g.H, g.V, g.H * 2, kBK, kBNHalf))
     return BGPO_ERR_CUDA;
   GemmArgs ga;
   ga.g = g;
-  ga.num_sms = sms;
+  ga.num_pairs = gemm_num_pairs(sms);
   ga.j = j;
   ga.coef = nullptr;
   ga.dW = nullptr;
@@ -219,7 +221,7 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
   }
   {
     TraceScope ts(prob->trace, KID_LMHEAD_FWD, s);
-    if (launch_gemm(GEMM_FWD, map_xm, map_w, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_gemm(GEMM_FWD, map_xm, map_w, map_xm, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_LSE_COMBINE, s);
@@ -272,34 +274,43 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   const WsPtrs w = ws_pointers(ws, L);
 
   CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xm_mn;
+  CUtensorMap map_dz_st, map_dxp_st, map_dw_red;
+  const uint64_t dxp_rows = (uint64_t)dxp_row_block_cap(g) * kPairM;
   if (!map_2d(&map_xm_k, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
-      !map_2d(&map_w_k, W, g.H, g.V, g.H * 2, kBK, kBN) ||
+      !map_2d(&map_w_k, W, g.H, g.V, g.H * 2, kBK, kBNHalf) ||
       !map_2d(&map_dz_k, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, kBK, kBM) ||
       !map_2d(&map_w_mn, W, g.H, g.V, g.H * 2, 64, kBK) ||
       !map_2d(&map_dz_mn, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, kBK) ||
-      !map_2d(&map_xm_mn, w.xm, g.H, g.m_pad, g.H * 2, 64, kBK))
+      !map_2d(&map_xm_mn, w.xm, g.H, g.m_pad, g.H * 2, 64, kBK) ||
+      // epilogue destinations: 32-row sub-tiles of 128 bytes
+      !map_2d(&map_dz_st, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, 32) ||
+      !map_2d(&map_dxp_st, w.dxp, g.H, dxp_rows, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32) ||
+      !map_2d(&map_dw_red, dW, g.H, g.V, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32))
     return BGPO_ERR_CUDA;
   GemmArgs ga;
   ga.g = g;
-  ga.num_sms = sms;
+  ga.num_pairs = gemm_num_pairs(sms);
   ga.j = j;
   ga.coef = coef;
   ga.dW = dW;
   {
     TraceScope ts(prob->trace, KID_LMHEAD_DZ, s);
-    if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, map_dz_st, ga, w, s) != cudaSuccess)
+      return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_DX_GEMM, s);
-    if (launch_gemm(GEMM_DX, map_dz_k, map_w_mn, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_gemm(GEMM_DX, map_dz_k, map_w_mn, map_dxp_st, ga, w, s) != cudaSuccess)
+      return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_DX_REDUCE, s);
-    if (launch_dx_reduce(g, j, sms, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_dx_reduce(g, j, ga.num_pairs, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_DW_GEMM, s);
-    if (launch_gemm(GEMM_DW, map_dz_mn, map_xm_mn, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_gemm(GEMM_DW, map_dz_mn, map_xm_mn, map_dw_red, ga, w, s) != cudaSuccess)
+      return BGPO_ERR_CUDA;
   }
   return BGPO_OK;
 }

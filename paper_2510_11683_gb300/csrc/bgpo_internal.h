@@ -44,7 +44,7 @@ cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, flo
 cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
                                 const float* ell_old, const float* A, float* coef_out,
                                 float* g_out, const WsPtrs& w, cudaStream_t s);
-cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_sms, const WsPtrs& w,
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_pairs, const WsPtrs& w,
                              float* dX, cudaStream_t s);
 cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
                                    cudaStream_t s);
@@ -54,13 +54,21 @@ enum GemmKind : int { GEMM_FWD = 0, GEMM_DZ = 1, GEMM_DX = 2, GEMM_DW = 3 };
 
 struct GemmArgs {
   Geometry g;
-  int num_sms;
+  int num_pairs;      // CTA pairs launched (gemm_num_pairs)
   int32_t j;
   const float* coef;  // GEMM_DZ: per-sequence dL/dl
   float* dW;          // GEMM_DW: accumulated weight gradient [V, H]
 };
 
+// CTA pairs the GEMM kernels run as: the 2-CTA clusters that fit on the
+// device at once (at most num_sms / 2), so that every pair of the persistent
+// grid is resident.
+int gemm_num_pairs(int num_sms);
+
+// map_a / map_b: the operand tiles; map_c: the epilogue's destination (dZ for
+// GEMM_DZ, the split-K partials for GEMM_DX, dW for GEMM_DW; unused by GEMM_FWD).
 cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorMap& map_b,
-                        const GemmArgs& a, const WsPtrs& w, cudaStream_t s);
+                        const CUtensorMap& map_c, const GemmArgs& a, const WsPtrs& w,
+                        cudaStream_t s);
 
 }  // namespace bgpo

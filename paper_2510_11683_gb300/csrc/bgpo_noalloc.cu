@@ -174,17 +174,17 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   a.mask_out = nullptr;
   CUtensorMap map_xm, map_w;
   if (!encode_map(&map_xm, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
-      !encode_map(&map_w, W, g.H, g.V, g.H * 2, kBK, kBN))
+      !encode_map(&map_w, W, g.H, g.V, g.H * 2, kBK, kBNHalf))
     return BGPO_ERR_CUDA;
   GemmArgs ga;
   ga.g = g;
-  ga.num_sms = sms;
+  ga.num_pairs = gemm_num_pairs(sms);
   ga.j = j;
   ga.coef = nullptr;
   ga.dW = nullptr;
   if (launch_mask_compact(a, w, s) != cudaSuccess ||
       launch_gather(g, j, X, Y, w, s) != cudaSuccess ||
-      launch_gemm(GEMM_FWD, map_xm, map_w, ga, w, s) != cudaSuccess ||
+      launch_gemm(GEMM_FWD, map_xm, map_w, map_xm, ga, w, s) != cudaSuccess ||
       launch_lse_combine(g, j, w, s) != cudaSuccess ||
       launch_seq_reduce(g, j, w, ell_out, s) != cudaSuccess)
     return BGPO_ERR_CUDA;

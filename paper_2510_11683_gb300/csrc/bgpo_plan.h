@@ -13,18 +13,28 @@
 
 namespace bgpo {
 
-// ---- GEMM tile geometry (one CTA computes a 128 x 256 fp32 tile in TMEM) ----
-constexpr int kBM = 128;         // rows per tile = TMEM lanes
+// ---- GEMM tile geometry ---------------------------------------------------------
+// A pair of CTAs (a 2-CTA cluster) computes one 256 x 256 fp32 tile with
+// tcgen05.mma.cta_group::2: each CTA holds 128 rows of A, 128 of the 256 B
+// columns and 128 accumulator rows in its own TMEM.
+constexpr int kBM = 128;         // accumulator rows per CTA = TMEM lanes
+constexpr int kPairM = 256;      // rows per pair tile
 constexpr int kBN = 256;         // columns per tile = TMEM columns per accumulator
+constexpr int kBNHalf = 128;     // B columns staged by each CTA of the pair
 constexpr int kBK = 64;          // K per pipeline stage: one 128-byte swizzle row of bf16
 constexpr int kUmmaK = 16;       // K of one tcgen05.mma kind::f16 instruction
-constexpr int kStages = 4;       // TMA -> MMA pipeline depth
+constexpr int kStages = 6;       // TMA -> MMA pipeline depth
 constexpr int kMaxSplits = 16;   // split-K limit of the dX GEMM
 
-constexpr uint32_t kTileABytes = kBM * kBK * 2;   // 16 KB
-constexpr uint32_t kTileBBytes = kBN * kBK * 2;   // 32 KB
+constexpr uint32_t kTileABytes = kBM * kBK * 2;       // 16 KB per CTA
+constexpr uint32_t kTileBBytes = kBNHalf * kBK * 2;   // 16 KB per CTA
 constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
-constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /*barriers*/ + 1024 /*align*/;
+// Epilogue staging: each of the 4 epilogue warps double-buffers one 32-row x
+// 128-byte sub-tile (32 fp32 or 64 bf16 columns) for its TMA stores.
+constexpr uint32_t kEpiBufBytes = 32 * 128;
+constexpr uint32_t kEpiBytes = 4 * 2 * kEpiBufBytes;   // 32 KB
+constexpr uint32_t kGemmSmemBytes =
+    kStages * kStageBytes + kEpiBytes + 1024 /*barriers*/ + 1024 /*align*/;
 
 // ---- kernel ids (trace + device error "where") --------------------------------
 enum KernelId : int32_t {
@@ -45,14 +55,15 @@ enum KernelId : int32_t {
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 BGPO_HD int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 
-// Split-K count of the dX GEMM (K = vocabulary) for `mb` row blocks times
-// `tiles_n` column tiles on `num_sms` SMs: the smallest s whose wave-quantised
-// time ceil(tiles*s/sms)/s is within 8% of the ideal tiles/sms, else the best s.
-// s * mb never exceeds `row_block_cap`, which bounds the partial buffer
-// independently of the SM count.
-BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_sms, int64_t k_blocks,
+// Split-K count of the dX GEMM (K = vocabulary) for `mb` pair row blocks times
+// `tiles_n` column tiles on `num_pairs` CTA pairs: the smallest s whose
+// wave-quantised time ceil(tiles*s/pairs)/s is within 8% of the ideal
+// tiles/pairs, else the best s. s * mb never exceeds `row_block_cap`, which
+// bounds the partial buffer independently of the SM count.
+BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_pairs, int64_t k_blocks,
                       int64_t row_block_cap) {
   const int64_t tiles_mn = mb * tiles_n;
+  const int num_sms = num_pairs;
   if (tiles_mn <= 0 || num_sms <= 0) return 1;
   int64_t smax = kMaxSplits;
   if (k_blocks < smax) smax = k_blocks > 0 ? k_blocks : 1;
@@ -72,7 +83,7 @@ BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_sms, int64_t k_blocks
 struct Geometry {
   int64_t B, P, R, H, V;
   int64_t m_cap;      // B * R: most masked rows a sample can have
-  int64_t m_pad;      // m_cap rounded up to a tile of rows
+  int64_t m_pad;      // m_cap rounded up to a pair tile of rows
   int64_t v_pad;      // V rounded up to 64 (row pitch of the dZ buffer)
   int64_t n_vt;       // vocabulary tiles of kBN columns
   int64_t tiles_h;    // hidden-size tiles of kBN columns
@@ -83,7 +94,7 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
   Geometry g;
   g.B = B; g.P = P; g.R = R; g.H = H; g.V = V;
   g.m_cap = B * R;
-  g.m_pad = round_up(g.m_cap, kBM);
+  g.m_pad = round_up(g.m_cap, kPairM);
   g.v_pad = round_up(V, 64);
   g.n_vt = ceil_div(V, kBN);
   g.tiles_h = ceil_div(H, kBN);
@@ -113,9 +124,10 @@ struct WsLayout {
 
 BGPO_HD size_t align_ws(size_t x) { return (x + 1023) & ~(size_t)1023; }
 
-// Row blocks the split-K partial buffer holds: enough for every split choice.
+// Pair row blocks (256 rows) the split-K partial buffer holds: enough for every
+// split choice.
 BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
-  const int64_t mb_max = g.m_pad / kBM;
+  const int64_t mb_max = g.m_pad / kPairM;
   return mb_max > kMaxSplits ? mb_max : kMaxSplits;
 }
 
@@ -134,7 +146,7 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g) {
   L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
   L.dz = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.v_pad);
-  L.dxp_elems = (size_t)dxp_row_block_cap(g) * kBM * (size_t)g.H;
+  L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;
   L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
   L.total = o;
   return L;

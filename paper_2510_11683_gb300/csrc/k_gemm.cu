@@ -1,12 +1,20 @@
 // The four LM-head contractions of the BGPO ELBO path on sm_103a tensor cores.
 //
-// Each is a persistent, warp-specialised kernel computing 128 x 256 fp32 tiles:
-//   warp 0      TMA producer: 128-byte-swizzled bf16 tiles into a 4-stage ring
-//   warp 1      TMEM owner + MMA issuer: tcgen05.mma kind::f16 (M=128, N=256,
-//               K=16) into one of two TMEM accumulators (2 x 256 columns)
-//   warps 2-5   epilogue: tcgen05.ld of the accumulator (thread = tile row),
-//               fused per-kind epilogue, accumulator handed back to the MMA warp
-// so the epilogue of tile n overlaps the main loop of tile n+1.
+// Each is a persistent, warp-specialised kernel launched as 2-CTA clusters. A
+// CTA pair computes 256 x 256 fp32 tiles with tcgen05.mma.cta_group::2: CTA r
+// of the pair stages rows [128 r, 128 r + 128) of the A tile and columns
+// [128 r, 128 r + 128) of the B tile, and holds accumulator rows
+// [128 r, 128 r + 128) in its TMEM. Roles in each CTA (192 threads):
+//   warp 0      TMA producer: 128-byte-swizzled bf16 boxes into a 6-stage ring
+//               of 32 KB; every copy of both CTAs completes on the even CTA's
+//               "full" barrier, which the even CTA alone arms with both CTAs'
+//               transaction bytes (a negative transaction count in between is
+//               allowed)
+//   warp 1      TMEM allocation (pair, 512 columns = two accumulators); in the
+//               even CTA also the MMA issuer (M = 256, N = 256, K = 16)
+//   warps 2-5   epilogue: tcgen05.ld of this CTA's accumulator rows, fused
+//               per-kind epilogue, TMA stores / reductions from shared memory
+// The epilogue of tile n overlaps the main loop of tile n+1.
 //
 // Kinds (Xm = gathered masked hidden states [M, H], W = LM head [V, H]):
 //   GEMM_FWD  z = Xm W^T; epilogue: online max / sum-exp per (row, vocab tile)
@@ -15,11 +23,13 @@
 //   GEMM_DZ   z = Xm W^T recomputed; epilogue: dz = w_r (onehot - e^{z - lse})
 //             stored as bf16 (gradient of Eq. 4 weighted by Eq. 13's dL/dl).
 //   GEMM_DX   dXm = dZ W (K = vocabulary, split-K partials in fp32).
-//   GEMM_DW   dW += dZ^T Xm (K = masked rows), fp32 read-modify-write.
+//   GEMM_DW   dW += dZ^T Xm (K = masked rows), fp32 TMA reduce-add.
 //
 // Every wait is bounded (time and polls); a wait that runs out sets the
-// workspace error word to BGPO_ERR_TIMEOUT and the CTA drains and exits.
+// workspace error word to BGPO_ERR_TIMEOUT and both CTAs drain and exit.
 #include <math.h>
+
+#include <mutex>
 
 #include "bgpo_device.cuh"
 #include "bgpo_internal.h"
@@ -34,10 +44,11 @@ constexpr int32_t kStatusTimeout = 8;     // BGPO_ERR_TIMEOUT
 constexpr int kThreads = 192;             // 6 warps
 constexpr uint32_t kTmemCols = 2 * kBN;   // two accumulators
 constexpr uint32_t kMnChunkBytes = 64 * 64 * 2;   // one 64 x 64 bf16 TMA box (MN-major)
+constexpr uint16_t kBothCtas = 0x3;
 
 struct GemmParams {
   Geometry g;
-  int num_sms;
+  int num_pairs;
   int32_t j;
   WsPtrs w;
   const float* coef;
@@ -58,20 +69,20 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M) {
   Work w;
   w.splits = 1;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
-    w.tiles_m = ceil_div(M, kBM);
+    w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = p.g.n_vt;
     w.kb_total = p.g.H / kBK;
     w.units = w.tiles_m * w.tiles_n;
   } else if (KIND == GEMM_DX) {
-    w.tiles_m = ceil_div(M, kBM);
+    w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = p.g.tiles_h;
     w.kb_total = p.g.kb_v;
-    w.splits = w.tiles_m > 0 ? dx_splits(w.tiles_m, w.tiles_n, p.num_sms, w.kb_total,
+    w.splits = w.tiles_m > 0 ? dx_splits(w.tiles_m, w.tiles_n, p.num_pairs, w.kb_total,
                                          dxp_row_block_cap(p.g))
                              : 1;
     w.units = w.tiles_m * w.tiles_n * w.splits;
   } else {  // GEMM_DW
-    w.tiles_m = ceil_div(p.g.V, kBM);
+    w.tiles_m = ceil_div(p.g.V, kPairM);
     w.tiles_n = p.g.tiles_h;
     w.kb_total = ceil_div(M, kBK);
     w.units = M > 0 ? w.tiles_m * w.tiles_n : 0;
@@ -90,6 +101,7 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
     t.kb0 = 0;
     t.kb_n = (int32_t)w.kb_total;
   } else if (KIND == GEMM_DX) {
+    // consecutive units share a column block of W
     const int64_t per_split = w.tiles_m * w.tiles_n;
     t.split = (int32_t)(u / per_split);
     const int64_t rem = u % per_split;
@@ -115,41 +127,55 @@ struct Majors {
   static constexpr bool b_mn = (KIND == GEMM_DX || KIND == GEMM_DW);
 };
 
-// Issues the TMA loads of one pipeline stage; returns the bytes they deliver.
+// Bytes this CTA's copies deliver for one stage of unit t (boxes that would lie
+// wholly outside the operand are not issued; their MMA outputs are discarded).
 template <int KIND>
-__device__ __forceinline__ uint32_t load_stage(const GemmParams& p, const CUtensorMap* ma,
-                                               const CUtensorMap* mb, uint32_t sa, uint32_t sb,
-                                               uint32_t bar, const Unit& t, int32_t kb) {
+__device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit& t, uint32_t rank) {
+  const int32_t a0 = t.m_blk * kPairM + (int32_t)rank * kBM;
+  const int32_t b0 = t.n_blk * kBN + (int32_t)rank * kBNHalf;
   uint32_t bytes = 0;
   if (!Majors<KIND>::a_mn) {
-    tma_load_2d(sa, ma, bar, kb * kBK, t.m_blk * kBM);
     bytes += kTileABytes;
   } else {
-    // dZ^T tile: 2 boxes of 64 vocabulary columns x 64 masked rows
-#pragma unroll
-    for (int c = 0; c < kBM / 64; ++c) {
-      const int32_t v = t.m_blk * kBM + c * 64;
-      if (v < p.g.v_pad) {
-        tma_load_2d(sa + c * kMnChunkBytes, ma, bar, v, kb * kBK);
-        bytes += kMnChunkBytes;
-      }
-    }
+    for (int c = 0; c < kBM / 64; ++c)
+      if (a0 + c * 64 < p.g.v_pad) bytes += kMnChunkBytes;
   }
   if (!Majors<KIND>::b_mn) {
-    tma_load_2d(sb, mb, bar, kb * kBK, t.n_blk * kBN);
-    bytes += kTileBBytes;
+    if (b0 < p.g.V) bytes += kTileBBytes;
   } else {
-    // W (GEMM_DX) or Xm (GEMM_DW) tile: 4 boxes of 64 hidden columns x 64 K rows
-#pragma unroll
-    for (int c = 0; c < kBN / 64; ++c) {
-      const int32_t h = t.n_blk * kBN + c * 64;
-      if (h < p.g.H) {
-        tma_load_2d(sb + c * kMnChunkBytes, mb, bar, h, kb * kBK);
-        bytes += kMnChunkBytes;
-      }
-    }
+    for (int c = 0; c < kBNHalf / 64; ++c)
+      if (b0 + c * 64 < p.g.H) bytes += kMnChunkBytes;
   }
   return bytes;
+}
+
+// Issues this CTA's TMA loads of one stage; they complete on `cbar`, the even
+// CTA's full barrier (shared::cluster address).
+template <int KIND>
+__device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMap* ma,
+                                           const CUtensorMap* mb, uint32_t sa, uint32_t sb,
+                                           uint32_t cbar, const Unit& t, int32_t kb,
+                                           uint32_t rank) {
+  const int32_t a0 = t.m_blk * kPairM + (int32_t)rank * kBM;
+  const int32_t b0 = t.n_blk * kBN + (int32_t)rank * kBNHalf;
+  if (!Majors<KIND>::a_mn) {
+    tma_load_2d_pair(sa, ma, cbar, kb * kBK, a0);
+  } else {
+    // dZ^T rows of this CTA: 2 boxes of 64 vocabulary columns x 64 masked rows
+#pragma unroll
+    for (int c = 0; c < kBM / 64; ++c)
+      if (a0 + c * 64 < p.g.v_pad)
+        tma_load_2d_pair(sa + c * kMnChunkBytes, ma, cbar, a0 + c * 64, kb * kBK);
+  }
+  if (!Majors<KIND>::b_mn) {
+    if (b0 < p.g.V) tma_load_2d_pair(sb, mb, cbar, kb * kBK, b0);
+  } else {
+    // W (GEMM_DX) or Xm (GEMM_DW) columns of this CTA: 2 boxes of 64 x 64
+#pragma unroll
+    for (int c = 0; c < kBNHalf / 64; ++c)
+      if (b0 + c * 64 < p.g.H)
+        tma_load_2d_pair(sb + c * kMnChunkBytes, mb, cbar, b0 + c * 64, kb * kBK);
+  }
 }
 
 __device__ __forceinline__ float bits_f(uint32_t v) { return __uint_as_float(v); }
@@ -159,13 +185,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// ---- epilogues: one thread per accumulator row ----------------------------------
+// ---- epilogues: one thread per accumulator row; row0 = first row of the warp --------
 
 // GEMM_FWD: per (row, vocab tile) the pair (max z, sum e^{z - max}) and, in the
 // tile holding y_r, the target logit z_{r, y_r}.
-__device__ __forceinline__ void epi_fwd(const GemmParams& p, int32_t M, const Unit& t, int row,
-                                        uint32_t tb) {
-  const int64_t r = (int64_t)t.m_blk * kBM + row;
+__device__ __forceinline__ void epi_fwd(const GemmParams& p, int32_t M, const Unit& t,
+                                        int64_t row0, int lane, uint32_t tb) {
+  const int64_t r = row0 + lane;
   const bool valid = r < M;
   const int32_t y = valid ? p.w.tgt[r] : -1;
   const int32_t v0 = t.n_blk * kBN;
@@ -202,11 +228,52 @@ __device__ __forceinline__ void epi_fwd(const GemmParams& p, int32_t M, const Un
   }
 }
 
+// Epilogue staging of one warp: two 32-row x 128-byte buffers in the 128-byte
+// swizzled layout the TMA tensor maps use (16-byte chunk q of row r stored at
+// chunk q ^ (r & 7)), so that 32 lanes writing one row each hit 8 bank groups.
+struct EpiStage {
+  uint32_t base;   // shared address of this warp's first buffer (1024-aligned)
+  int buf;         // buffer the next sub-tile goes to
+
+  // Returns the shared address of a buffer free for writing: the bulk group
+  // that last read it (two sub-tiles ago) has finished reading.
+  __device__ __forceinline__ uint32_t acquire(int lane) {
+    if (lane == 0) bulk_wait_group_read<1>();
+    __syncwarp();
+    return base + (uint32_t)buf * kEpiBufBytes;
+  }
+  // Hands the written buffer to lane 0, which issues the bulk copy `issue`.
+  template <class Issue>
+  __device__ __forceinline__ void release(int lane, uint32_t sbuf, Issue issue) {
+    fence_proxy_async_shared();
+    __syncwarp();
+    if (lane == 0) {
+      issue(sbuf);
+      bulk_commit_group();
+    }
+    buf ^= 1;
+  }
+};
+
+// Writes 8 16-byte chunks (one 128-byte row of the sub-tile) for row `lane`.
+__device__ __forceinline__ void stage_row(uint32_t sbuf, int lane, const uint4 (&chunk)[8]) {
+  const uint32_t row = sbuf + (uint32_t)lane * 128u;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const uint32_t a = row + (uint32_t)((q ^ (lane & 7)) * 16);
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(chunk[q].x),
+                 "r"(chunk[q].y), "r"(chunk[q].z), "r"(chunk[q].w)
+                 : "memory");
+  }
+}
+
 // GEMM_DZ: dz_{r,v} = w_r (1[v = y_r] - e^{z_{r,v} - lse_r}) as bf16, zero for
-// rows >= M and vocabulary columns >= V (the dZ row pitch is v_pad).
-__device__ __forceinline__ void epi_dz(const GemmParams& p, int32_t M, const Unit& t, int row,
-                                       uint32_t tb) {
-  const int64_t r = (int64_t)t.m_blk * kBM + row;
+// rows >= M and vocabulary columns >= V; 64-column sub-tiles leave through TMA
+// stores into dZ [m_pad, v_pad].
+__device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
+                                       const Unit& t, int64_t row0, int lane, uint32_t tb,
+                                       EpiStage& st) {
+  const int64_t r = row0 + lane;
   const bool valid = r < M;
   float w = 0.f, lse_l2 = 0.f;
   int32_t y = -1;
@@ -218,80 +285,83 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, int32_t M, const Uni
   }
   const int32_t v0 = t.n_blk * kBN;
   const int32_t V = (int32_t)p.g.V;
-  __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.w.dz) + r * p.g.v_pad + v0;
 #pragma unroll 1
-  for (int c = 0; c < kBN / 32; ++c) {
-    const int32_t col0 = v0 + c * 32;
+  for (int c = 0; c < kBN / 64; ++c) {
+    const int32_t col0 = v0 + c * 64;
     if (col0 >= p.g.v_pad) break;  // warp-uniform
-    uint32_t raw[32];
-    tmem_ld_32x32b_x32(tb + c * 32, raw);
-    tmem_ld_wait();
-    uint32_t packed[16];
+    uint4 chunk[8];
 #pragma unroll
-    for (int k = 0; k < 32; k += 2) {
-      float d[2];
+    for (int h = 0; h < 2; ++h) {
+      uint32_t raw[32];
+      tmem_ld_32x32b_x32(tb + c * 64 + h * 32, raw);
+      tmem_ld_wait();
+      uint32_t packed[16];
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int32_t col = col0 + k + e;
-        const float pr = exp2f(fmaf(bits_f(raw[k + e]), kLog2e, -lse_l2));
-        const float v = w * ((col == y ? 1.f : 0.f) - pr);
-        d[e] = (valid && col < V) ? v : 0.f;
+      for (int k = 0; k < 32; k += 2) {
+        float d[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int32_t col = col0 + h * 32 + k + e;
+          const float pr = exp2f(fmaf(bits_f(raw[k + e]), kLog2e, -lse_l2));
+          const float v = w * ((col == y ? 1.f : 0.f) - pr);
+          d[e] = (valid && col < V) ? v : 0.f;
+        }
+        packed[k / 2] = pack_bf16x2(d[0], d[1]);
       }
-      packed[k / 2] = pack_bf16x2(d[0], d[1]);
-    }
-    uint4* o = reinterpret_cast<uint4*>(dst + c * 32);
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
-      o[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+      for (int q = 0; q < 4; ++q)
+        chunk[h * 4 + q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
+                                      packed[4 * q + 3]);
+    }
+    const uint32_t sbuf = st.acquire(lane);
+    stage_row(sbuf, lane, chunk);
+    st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, col0, (int32_t)row0); });
   }
 }
 
-// GEMM_DX: fp32 partial of split s for masked row r.
-__device__ __forceinline__ void epi_dx(const GemmParams& p, int32_t M, const Work& wk, const Unit& t,
-                                       int row, uint32_t tb) {
-  const int64_t r = (int64_t)t.m_blk * kBM + row;
+// GEMM_DX: fp32 partial of split s, rows [split * tiles_m * 256 + r] of the
+// partial buffer, 32-column sub-tiles through TMA stores (rows >= M hold zeros).
+__device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* map_c,
+                                       const Work& wk, const Unit& t, int64_t row0, int lane,
+                                       uint32_t tb, EpiStage& st) {
   const int32_t h0 = t.n_blk * kBN;
-  const int64_t split_stride = wk.tiles_m * kBM * p.g.H;
-  float* dst = p.w.dxp + t.split * split_stride + r * p.g.H + h0;
+  const int32_t prow0 = (int32_t)(t.split * wk.tiles_m * kPairM + row0);
 #pragma unroll 1
   for (int c = 0; c < kBN / 32; ++c) {
     if (h0 + c * 32 >= p.g.H) break;  // warp-uniform
     uint32_t raw[32];
     tmem_ld_32x32b_x32(tb + c * 32, raw);
     tmem_ld_wait();
-    if (r < M) {
-      float4* o = reinterpret_cast<float4*>(dst + c * 32);
+    uint4 chunk[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        o[q] = make_float4(bits_f(raw[4 * q]), bits_f(raw[4 * q + 1]), bits_f(raw[4 * q + 2]),
-                           bits_f(raw[4 * q + 3]));
-    }
+    for (int q = 0; q < 8; ++q)
+      chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
+    const uint32_t sbuf = st.acquire(lane);
+    stage_row(sbuf, lane, chunk);
+    st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, h0 + c * 32, prow0); });
   }
 }
 
-// GEMM_DW: dW[v, h] += acc for vocabulary row v < V.
-__device__ __forceinline__ void epi_dw(const GemmParams& p, const Unit& t, int row, uint32_t tb) {
-  const int64_t v = (int64_t)t.m_blk * kBM + row;
+// GEMM_DW: dW[v, h] += acc through TMA reduce-add of 32 x 32 fp32 sub-tiles
+// (the read-modify-write happens at L2; vocabulary rows >= V are clipped).
+__device__ __forceinline__ void epi_dw(const GemmParams& p, const CUtensorMap* map_c, const Unit& t,
+                                       int64_t row0, int lane, uint32_t tb, EpiStage& st) {
   const int32_t h0 = t.n_blk * kBN;
-  float* dst = p.dW + v * p.g.H + h0;
+  if (row0 >= p.g.V) return;  // this warp's rows all lie past the vocabulary (warp-uniform)
 #pragma unroll 1
   for (int c = 0; c < kBN / 32; ++c) {
     if (h0 + c * 32 >= p.g.H) break;  // warp-uniform
     uint32_t raw[32];
     tmem_ld_32x32b_x32(tb + c * 32, raw);
     tmem_ld_wait();
-    if (v < p.g.V) {
-      float4* o = reinterpret_cast<float4*>(dst + c * 32);
+    uint4 chunk[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        float4 a = o[q];
-        a.x += bits_f(raw[4 * q]);
-        a.y += bits_f(raw[4 * q + 1]);
-        a.z += bits_f(raw[4 * q + 2]);
-        a.w += bits_f(raw[4 * q + 3]);
-        o[q] = a;
-      }
-    }
+    for (int q = 0; q < 8; ++q)
+      chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
+    const uint32_t sbuf = st.acquire(lane);
+    stage_row(sbuf, lane, chunk);
+    st.release(lane, sbuf,
+               [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, (int32_t)row0); });
   }
 }
 
@@ -303,20 +373,28 @@ __device__ __forceinline__ int32_t kernel_id() {
                           : KID_DW_GEMM;
 }
 
+// Sets the abort flag of both CTAs of the pair.
+__device__ __forceinline__ void raise_abort(volatile int* abort_flag, uint32_t peer) {
+  *abort_flag = 1;
+  const uint32_t remote = map_to_cta(smem_addr(const_cast<int*>(abort_flag)), peer);
+  asm volatile("st.relaxed.cluster.shared::cluster.u32 [%0], %1;" ::"r"(remote), "r"(1) : "memory");
+}
+
 template <int KIND>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-           const GemmParams p) {
+           const __grid_constant__ CUtensorMap map_c, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* s_a = smem;
   uint8_t* s_b = smem + kStages * kTileABytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_b + kStages * kTileBBytes);
-  uint64_t* full = bars;                      // [kStages] TMA -> MMA
-  uint64_t* empty = bars + kStages;           // [kStages] MMA -> TMA
-  uint64_t* tfull = bars + 2 * kStages;       // [2] MMA -> epilogue
-  uint64_t* tempty = bars + 2 * kStages + 2;  // [2] epilogue -> MMA
+  uint8_t* s_epi = s_b + kStages * kTileBBytes;   // 4 warps x 2 staging buffers
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_epi + kEpiBytes);
+  uint64_t* full = bars;                      // [kStages] TMA (both CTAs) -> MMA; even CTA's
+  uint64_t* empty = bars + kStages;           // [kStages] MMA -> TMA of each CTA
+  uint64_t* tfull = bars + 2 * kStages;       // [2] MMA -> epilogue of each CTA
+  uint64_t* tempty = bars + 2 * kStages + 2;  // [2] epilogues (both CTAs) -> MMA; even CTA's
   uint64_t* done = bars + 2 * kStages + 4;    // MMA drain on abort
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 5);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -324,6 +402,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: even CTA (issues the MMAs), 1: its peer
+  const uint32_t peer = rank ^ 1u;
+  const int64_t pair = blockIdx.x >> 1;
+  const int64_t num_pairs = gridDim.x >> 1;
   int32_t* err = p.w.err;
 
   int32_t M = 0;
@@ -333,16 +415,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     set_device_error(err, kStatusInvalidArg, kernel_id<KIND>() * 16 + 1);
   }
   const Work wk = make_work<KIND>(p, M);
-  if ((int64_t)blockIdx.x >= wk.units) return;  // whole CTA, before any allocation
+  if (pair >= wk.units) return;  // both CTAs of the pair, before any allocation
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(smem_addr(&full[s]), 1);
-      mbar_init(smem_addr(&empty[s]), 1);
+      mbar_init(smem_addr(&full[s]), 1);    // the even CTA's arrive.expect_tx
+      mbar_init(smem_addr(&empty[s]), 1);   // one multicast commit
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_addr(&tfull[a]), 1);
-      mbar_init(smem_addr(&tempty[a]), 4 * 32);
+      mbar_init(smem_addr(&tempty[a]), 2 * 4);   // 4 epilogue warps in each CTA
     }
     mbar_init(smem_addr(done), 1);
     *abort_flag = 0;
@@ -352,70 +434,63 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&map_a);
     tma_prefetch_map(&map_b);
+    if (KIND != GEMM_FWD) tma_prefetch_map(&map_c);
   }
   if (warp == 1) {
-    tmem_alloc(smem_addr(tmem_slot), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_addr(tmem_slot), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
+    // ---------------- TMA producer (both CTAs) ----------------
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      uint32_t armed = 0;  // bit s: stage s has copies that may still be in flight
-      for (int64_t u = blockIdx.x; u < wk.units && ok; u += gridDim.x) {
+      bool issued = false;
+      for (int64_t u = pair; u < wk.units && ok; u += num_pairs) {
         const Unit t = unit_of<KIND>(wk, u);
+        // the even CTA arms the transaction bytes of both CTAs' copies on its
+        // full barrier; the odd CTA's copies only complete_tx on it (a
+        // per-stage remote arrive from the odd CTA halved the throughput)
+        const uint32_t bytes =
+            rank == 0 ? stage_bytes<KIND>(p, t, 0) + stage_bytes<KIND>(p, t, 1) : 0u;
         for (int32_t kb = t.kb0; kb < t.kb0 + t.kb_n; ++kb) {
           if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1u, abort_flag)) { ok = false; break; }
-          const uint32_t bar = smem_addr(&full[stage]);
-          const uint32_t sa = smem_addr(s_a + stage * kTileABytes);
-          const uint32_t sb = smem_addr(s_b + stage * kTileBBytes);
-          // the expected byte count is armed before the copies that complete it
-          uint32_t bytes = 0;
-          if (!Majors<KIND>::a_mn) bytes += kTileABytes;
-          else
-            for (int c = 0; c < kBM / 64; ++c)
-              if (t.m_blk * kBM + c * 64 < p.g.v_pad) bytes += kMnChunkBytes;
-          if (!Majors<KIND>::b_mn) bytes += kTileBBytes;
-          else
-            for (int c = 0; c < kBN / 64; ++c)
-              if (t.n_blk * kBN + c * 64 < p.g.H) bytes += kMnChunkBytes;
-          mbar_arrive_expect_tx(bar, bytes);
-          load_stage<KIND>(p, &map_a, &map_b, sa, sb, bar, t, kb);
-          armed |= 1u << stage;
+          const uint32_t cbar = map_to_cta(smem_addr(&full[stage]), 0);
+          if (rank == 0) mbar_arrive_expect_tx(smem_addr(&full[stage]), bytes);
+          load_stage<KIND>(p, &map_a, &map_b, smem_addr(s_a + stage * kTileABytes),
+                           smem_addr(s_b + stage * kTileBBytes), cbar, t, kb, rank);
+          issued = true;
           if (++stage == kStages) { stage = 0; phase ^= 1u; }
         }
       }
       if (!ok) {
-        *abort_flag = 1;
+        raise_abort(abort_flag, peer);
         set_device_error(err, kStatusTimeout, kernel_id<KIND>() * 16 + 2);
-        // Let copies already issued land before the CTA exits: stage s was last
-        // armed in phase `phase` if s < stage, else in phase `phase ^ 1`.
-        for (int s = 0; s < kStages; ++s) {
-          if (!((armed >> s) & 1u)) continue;
-          const uint32_t ph = (s < stage) ? phase : (phase ^ 1u);
+        // let copies already issued land before this CTA can exit
+        if (issued) {
           const uint64_t t0 = globaltimer_ns();
-          while (!mbar_try_wait(smem_addr(&full[s]), ph) && globaltimer_ns() - t0 < 10000000ull) {
+          while (globaltimer_ns() - t0 < 2000000ull) {
           }
         }
       }
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, Majors<KIND>::a_mn, Majors<KIND>::b_mn);
+    // ---------------- MMA issuer (even CTA) ----------------
+    if (rank == 0 && lane == 0) {
+      constexpr uint32_t idesc =
+          idesc_bf16_f32(kPairM, kBN, Majors<KIND>::a_mn, Majors<KIND>::b_mn);
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
       int it = 0;
-      for (int64_t u = blockIdx.x; u < wk.units && ok; u += gridDim.x, ++it) {
+      for (int64_t u = pair; u < wk.units && ok; u += num_pairs, ++it) {
         const Unit t = unit_of<KIND>(wk, u);
         const int acc = it & 1;
         const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
@@ -433,32 +508,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                    : smem_desc_sw128(sa + k * 32, 16, 1024);
             const uint64_t bd = Majors<KIND>::b_mn ? smem_desc_sw128(sb + k * 2048, kMnChunkBytes, 1024)
                                                    : smem_desc_sw128(sb + k * 32, 16, 1024);
-            umma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
           issued = true;
-          umma_commit(smem_addr(&empty[stage]));  // frees the stage once these MMAs finish
+          // frees this stage in both CTAs once these MMAs have read it
+          umma_commit_pair(smem_addr(&empty[stage]), kBothCtas);
           if (++stage == kStages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        umma_commit(smem_addr(&tfull[acc]));  // accumulator ready for the epilogue
+        umma_commit_pair(smem_addr(&tfull[acc]), kBothCtas);  // accumulators ready
       }
       if (!ok) {
-        *abort_flag = 1;
+        raise_abort(abort_flag, peer);
         set_device_error(err, kStatusTimeout, kernel_id<KIND>() * 16 + 3);
         if (issued) {
-          umma_commit(smem_addr(done));
+          umma_commit_pair(smem_addr(done), 0x1);
           mbar_wait(smem_addr(done), 0, never);
         }
       }
     }
     __syncwarp();
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
+    // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
     const int quarter = warp & 3;  // TMEM lanes this warp may access: 32*quarter ..
-    const int row = quarter * 32 + lane;
+    EpiStage st;
+    st.base = smem_addr(s_epi + (uint32_t)(warp - 2) * 2u * kEpiBufBytes);
+    st.buf = 0;
     int it = 0;
     bool ok = true;
-    for (int64_t u = blockIdx.x; u < wk.units; u += gridDim.x, ++it) {
+    for (int64_t u = pair; u < wk.units; u += num_pairs, ++it) {
       const Unit t = unit_of<KIND>(wk, u);
       const int acc = it & 1;
       const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
@@ -466,53 +544,80 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN);
-      if (KIND == GEMM_FWD) epi_fwd(p, M, t, row, tb);
-      else if (KIND == GEMM_DZ) epi_dz(p, M, t, row, tb);
-      else if (KIND == GEMM_DX) epi_dx(p, M, wk, t, row, tb);
-      else epi_dw(p, t, row, tb);
+      const int64_t row0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM + quarter * 32;
+      if (KIND == GEMM_FWD) epi_fwd(p, M, t, row0, lane, tb);
+      else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, lane, tb, st);
+      else if (KIND == GEMM_DX) epi_dx(p, &map_c, wk, t, row0, lane, tb, st);
+      else epi_dw(p, &map_c, t, row0, lane, tb, st);
       tc_fence_before();
-      mbar_arrive(smem_addr(&tempty[acc]));
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(map_to_cta(smem_addr(&tempty[acc]), 0));
     }
+    // every bulk store / reduction of this warp has completed before exit
+    if (lane == 0) bulk_wait_group<0>();
+    __syncwarp();
     if (!ok) {
-      *abort_flag = 1;
+      raise_abort(abort_flag, peer);
       if (lane == 0) set_device_error(err, kStatusTimeout, kernel_id<KIND>() * 16 + 4);
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // no CTA of the pair still reads the other's shared memory
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
 template <int KIND>
-cudaError_t launch_kind(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p,
-                        cudaStream_t s) {
+cudaError_t launch_kind(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc,
+                        const GemmParams& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(k_gemm<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kGemmSmemBytes);
   if (e != cudaSuccess) return e;
-  k_gemm<KIND><<<p.num_sms, kThreads, kGemmSmemBytes, s>>>(ma, mb, p);
+  k_gemm<KIND><<<2 * p.num_pairs, kThreads, kGemmSmemBytes, s>>>(ma, mb, mc, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
+int gemm_num_pairs(int num_sms) {
+  static int cached = 0;
+  static std::once_flag once;
+  std::call_once(once, [num_sms] {
+    int clusters = 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)num_sms, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kGemmSmemBytes;
+    if (cudaFuncSetAttribute(k_gemm<GEMM_DX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kGemmSmemBytes) == cudaSuccess &&
+        cudaOccupancyMaxActiveClusters(&clusters, k_gemm<GEMM_DX>, &cfg) == cudaSuccess &&
+        clusters > 0)
+      cached = clusters;
+    else
+      cudaGetLastError();
+  });
+  const int half = num_sms / 2;
+  return (cached > 0 && cached < half) ? cached : half;
+}
+
 cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorMap& map_b,
-                        const GemmArgs& a, const WsPtrs& w, cudaStream_t s) {
+                        const CUtensorMap& map_c, const GemmArgs& a, const WsPtrs& w,
+                        cudaStream_t s) {
   GemmParams p;
   p.g = a.g;
-  p.num_sms = a.num_sms;
+  p.num_pairs = a.num_pairs;
   p.j = a.j;
   p.w = w;
   p.coef = a.coef;
   p.dW = a.dW;
   switch (kind) {
-    case GEMM_FWD: return launch_kind<GEMM_FWD>(map_a, map_b, p, s);
-    case GEMM_DZ: return launch_kind<GEMM_DZ>(map_a, map_b, p, s);
-    case GEMM_DX: return launch_kind<GEMM_DX>(map_a, map_b, p, s);
-    case GEMM_DW: return launch_kind<GEMM_DW>(map_a, map_b, p, s);
+    case GEMM_FWD: return launch_kind<GEMM_FWD>(map_a, map_b, map_c, p, s);
+    case GEMM_DZ: return launch_kind<GEMM_DZ>(map_a, map_b, map_c, p, s);
+    case GEMM_DX: return launch_kind<GEMM_DX>(map_a, map_b, map_c, p, s);
+    case GEMM_DW: return launch_kind<GEMM_DW>(map_a, map_b, map_c, p, s);
   }
   return cudaErrorInvalidValue;
 }

@@ -117,15 +117,15 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
 // ---------------------------------------------------------------------------
 // Gather of the masked rows' hidden states (the indicator of Eq. 4 selects
 // them): Xm[r] = X[b, P + i] with 16-byte vector copies, one warp per row.
-// Rows [M, round_up(M, 128)) are zero-filled so that the GEMM tiles and the
-// K padding of the dW GEMM read zeros.
+// Rows [M, round_up(M, 256)) are zero-filled so that the GEMM pair tiles and
+// the K padding of the dW GEMM read zeros.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_gather(Geometry g, int32_t j, const uint4* __restrict__ X,
                                                 const int32_t* __restrict__ Y, WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_GATHER);
   const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (r >= round_up(M, kBM)) return;
+  if (r >= round_up(M, kPairM)) return;
   const int64_t nvec = g.H / 8;
   uint4* dst = reinterpret_cast<uint4*>(w.xm) + r * nvec;
   if (r < M) {
@@ -221,14 +221,14 @@ __global__ void k_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const f
 // dX[b, i, :] += sum_s partial_s[r, :] over the split-K partials of the dX GEMM
 // (fixed split order; rows are unique within a sample, so no atomics).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, int num_sms, WsPtrs w,
+__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, int num_pairs, WsPtrs w,
                                                    float* __restrict__ dX) {
   const int32_t M = rows_of_sample(w.err, j, KID_DX_REDUCE);
   const int64_t r = blockIdx.x;
   if (r >= M) return;
-  const int64_t mb = ceil_div(M, kBM);
-  const int S = dx_splits(mb, g.tiles_h, num_sms, g.kb_v, dxp_row_block_cap(g));
-  const int64_t split_stride = mb * kBM * g.H / 4;
+  const int64_t mb = ceil_div(M, kPairM);
+  const int S = dx_splits(mb, g.tiles_h, num_pairs, g.kb_v, dxp_row_block_cap(g));
+  const int64_t split_stride = mb * kPairM * g.H / 4;
   const float4* src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
   float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)w.rows[r] * (g.H / 4);
   for (int64_t h = threadIdx.x; h < g.H / 4; h += blockDim.x) {
@@ -313,9 +313,9 @@ cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const 
   return cudaGetLastError();
 }
 
-cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_sms, const WsPtrs& w, float* dX,
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_pairs, const WsPtrs& w, float* dX,
                              cudaStream_t s) {
-  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, num_sms, w, dX);
+  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, num_pairs, w, dX);
   return cudaGetLastError();
 }
 

@@ -91,7 +91,7 @@ def test_workspace_independent_of_n_t(L, bg):
 
 def test_workspace_grows_with_rows_and_vocab(L, bg):
     a = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg)))
-    assert L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=8))) > a
+    assert L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=16))) > a
     assert L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, V=4096))) > a
 
 
