@@ -203,6 +203,32 @@ def config_of(wl):
 # native arm
 # ----------------------------------------------------------------------------------
 
+def aggregate_ranks(ms_local, tokens_local):
+    """Whole-job figures of a data-parallel run: the slowest rank's ms per step
+    and the masked tokens of all ranks (torch.distributed must be initialised
+    when the world is larger than one)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms_local, tokens_local
+    dev = torch.device("cuda", torch.cuda.current_device()) \
+        if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([ms_local], dtype=torch.float64, device=dev)
+    n = torch.tensor([tokens_local], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n.item())
+
+
+def shard_of(wl, rank, world):
+    """(data workload, b_offset) of `rank`: every rank owns its own B responses,
+    which are sequences [rank * B, (rank + 1) * B) of a world * B batch; draws use
+    the batch seed and the global sequence index, data draws a per-rank seed."""
+    if world == 1:
+        return wl, 0
+    return wl.with_(seed=wl.seed + 7919 * rank), rank * wl.B
+
+
 def kernel_sha():
     with open(os.path.join(ROOT, "paper_2510_11683_gb300", "csrc", "k_gemm.cu"), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()
@@ -230,14 +256,15 @@ def main():
         B.build()
     from synth import make_inputs
 
-    # weak scaling: every rank owns its own batch of responses (independent units)
-    wl_r = wl.with_(seed=wl.seed + 1000 * rank) if world > 1 else wl
-    inp_cpu = make_inputs(wl_r)
+    # weak scaling: every rank owns B responses of a world * B batch (no collective
+    # in the data path; the dW all-reduce of an optimiser step lies outside it)
+    wl_data, b_offset = shard_of(wl, rank, world)
+    inp_cpu = make_inputs(wl_data)
     inp = {k: (v.to(dev) if v is not None else None) for k, v in inp_cpu.items()}
     X, W, Y = inp["X"], inp["W"], inp["Y"]
     n_t, Bsz = wl.n_t, wl.B
 
-    prob = bg.problem_from(wl_r)
+    prob = bg.problem_from(wl, b_offset=b_offset)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     A = torch.empty(Bsz, dtype=torch.float32, device=dev)
@@ -279,7 +306,7 @@ def main():
     torch.cuda.synchronize()
 
     trace = bg.Trace(args.steps * n_t * 12 + 16)
-    prob_t = bg.problem_from(wl_r, trace=trace)
+    prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset)
     clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
     stream = torch.cuda.current_stream()
     e0 = torch.cuda.Event(enable_timing=True)
@@ -295,12 +322,7 @@ def main():
     torch.cuda.synchronize()
     barrier()
     clock_info = clocks.stop()
-    ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms, masked_all = aggregate_ranks(e0.elapsed_time(e1) / args.steps, masked_per_step)
     code, where = bg.get_device_error(ws)
     if code != 0:
         raise RuntimeError(f"device error {code} at {where}")
@@ -331,7 +353,7 @@ def main():
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
                 "flops_per_launch": dom_flops_per_launch, "avg_launch_ms": dom_avg_s * 1e3}
 
-    value = masked_per_step * world / (ms / 1e3)
+    value = masked_all / (ms / 1e3)
     exec_tflops = 4 * gemm_flops_per_step / (ms / 1e3) / 1e12
 
     out = {

@@ -87,8 +87,11 @@ typedef struct bgpo_trace bgpo_trace;
  *   n_t    MC samples per response, 1 <= n_t < 65536 (Eq. 5)
  *   G      group size used by bgpo_group_advantage (Eq. 18), >= 1
  *   t_mode BGPO_T_IID or BGPO_T_STRATIFIED
- *   seed   Philox4x64-10 key word 0; the draws of (b, j) depend on (seed, b, j) only
+ *   seed   Philox4x64-10 key word 0; the draws of (b, j) depend on (seed, b_offset + b, j)
  *   loss_scale  L_j = -loss_scale * g_j; Algorithm 1 uses 1/G
+ *   b_offset  global index of this batch's first sequence (>= 0). A data-parallel
+ *          shard holding sequences [b_offset, b_offset + B) of a larger batch
+ *          draws exactly the t and masks the whole batch would draw for them.
  *   trace  optional bgpo_trace* (NULL = off)
  * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
  * bgpo_workspace_bytes).
@@ -104,7 +107,7 @@ typedef struct bgpo_problem {
   int32_t t_mode;
   uint64_t seed;
   float loss_scale;
-  int32_t flags;       /* reserved, must be 0 */
+  int32_t b_offset;
   bgpo_trace* trace;
 } bgpo_problem;
 
@@ -116,7 +119,7 @@ const char* bgpo_status_string(bgpo_status status);
 
 /*
  * Host-only validation of a problem description (no CUDA call).
- * Returns BGPO_OK, BGPO_ERR_INVALID_ARG (NULL, bad t_mode, flags != 0,
+ * Returns BGPO_OK, BGPO_ERR_INVALID_ARG (NULL, bad t_mode, negative b_offset,
  * non-finite loss_scale) or BGPO_ERR_SHAPE.
  */
 bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
@@ -130,11 +133,12 @@ size_t bgpo_workspace_bytes(const bgpo_problem* prob);
 
 /*
  * Forward masking process for MC sample j (Sec. 2.1; Eq. 3, 5; Algorithm 1).
- * Draws t_{b,j} = T/D with Philox4x64-10 (key (seed, 0), counter (0, b, j, 1),
+ * Draws t_{b,j} = T/D with Philox4x64-10 (key (seed, 0), counter (0, b', j, 1)
+ * with b' = b_offset + b the global sequence index,
  * T = u24 + 1 and D = 2^24, or T = j 2^24 + u24 + 1 and D = n_t 2^24 when
  * stratified; u24 = top 24 bits of output word 0) and masks response position
  * i of sequence b iff u24_i * D < T * 2^24, where u24_i is the top 24 bits of
- * output word (i mod 4) of the block with counter (i / 4, b, j, 0). Prompt
+ * output word (i mod 4) of the block with counter (i / 4, b', j, 0). Prompt
  * positions are never masked. Compacts the masked positions into ascending
  * (b, i) order inside the workspace.
  *   j         sample index, 0 <= j < n_t

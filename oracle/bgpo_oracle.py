@@ -69,9 +69,11 @@ def mask_bit(u24, T, D):
     return int(int(u24) * int(D) < int(T) * TWO24)
 
 
-def sample_t_mask(seed, B, R, j, n_t, t_mode):
-    """Timesteps and response masks of MC sample j for all B sequences.
+def sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset=0):
+    """Timesteps and response masks of MC sample j for B sequences.
 
+    Sequence b of this batch has global index b_offset + b in the counters, so a
+    shard of a larger batch draws what the whole batch draws for those rows.
     Returns (T [B] int64, D int, t [B] float64, mask [B, R] uint8). Prompt
     positions are never masked (Sec. 2.1), so only the R response positions
     appear here.
@@ -79,10 +81,10 @@ def sample_t_mask(seed, B, R, j, n_t, t_mode):
     T = np.zeros(B, dtype=np.int64)
     D = None
     for b in range(B):
-        T[b], D = t_numerator(seed, b, j, n_t, t_mode)
+        T[b], D = t_numerator(seed, b_offset + b, j, n_t, t_mode)
     Q = (R + 3) // 4
     q = np.arange(Q, dtype=np.uint64)[None, :]
-    bb = np.arange(B, dtype=np.uint64)[:, None]
+    bb = (np.arange(B, dtype=np.uint64) + np.uint64(b_offset))[:, None]
     words = philox4x64_10_array(q, bb, np.uint64(j), np.uint64(STREAM_MASK), seed, 0)
     u = np.stack(words, axis=-1).reshape(B, Q * 4)[:, :R] >> np.uint64(U24_SHIFT)
     mask = mask_bit(u, T.astype(np.uint64)[:, None], D)
@@ -245,11 +247,11 @@ def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192):
 # Algorithm 1, inner loops: all n_t MC samples of one batch
 # ---------------------------------------------------------------------------
 
-def sample_masks(seed, B, R, n_t, t_mode):
+def sample_masks(seed, B, R, n_t, t_mode, b_offset=0):
     """(t [n_t, B], mask [n_t, B, R]) for every MC sample j."""
     ts, masks = [], []
     for j in range(n_t):
-        _, _, t, m = sample_t_mask(seed, B, R, j, n_t, t_mode)
+        _, _, t, m = sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset)
         ts.append(t)
         masks.append(m)
     return np.stack(ts), np.stack(masks)

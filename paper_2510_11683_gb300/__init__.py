@@ -25,21 +25,25 @@ def _torch():
     return torch
 
 
-def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None):
-    """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1)."""
+def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None,
+            b_offset=0):
+    """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1).
+
+    b_offset: global index of the first sequence (a data-parallel shard of a
+    larger batch draws the same t and masks as the whole batch would)."""
     p = BgpoProblem()
     p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
     p.seed = seed
     p.loss_scale = (1.0 / G if G > 0 else 1.0) if loss_scale is None else loss_scale
-    p.flags = 0
+    p.b_offset = b_offset
     p.trace = trace.handle if isinstance(trace, Trace) else trace
     return p
 
 
-def problem_from(wl, trace=None, loss_scale=None):
+def problem_from(wl, trace=None, loss_scale=None, b_offset=0):
     """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
     return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
-                   loss_scale=loss_scale, trace=trace)
+                   loss_scale=loss_scale, trace=trace, b_offset=b_offset)
 
 
 def validate_problem(prob):

@@ -53,12 +53,13 @@ struct TraceScope {
 bgpo_status check_problem(const bgpo_problem* p) {
   if (!p) return BGPO_ERR_INVALID_ARG;
   if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
-  if (p->flags != 0) return BGPO_ERR_INVALID_ARG;
+  if (p->b_offset < 0) return BGPO_ERR_INVALID_ARG;
   if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
   if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
   if ((int64_t)p->B * p->R > kMaxRows) return BGPO_ERR_SHAPE;
+  if ((int64_t)p->b_offset + p->B > (int64_t(1) << 31)) return BGPO_ERR_SHAPE;
   if ((int64_t)p->B * ((int64_t)p->P + p->R) * p->H > (int64_t(1) << 40)) return BGPO_ERR_SHAPE;
   return BGPO_OK;
 }
@@ -177,6 +178,7 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
   const WsPtrs w = ws_pointers(ws, L);
   MaskArgs a;
   a.seed = prob->seed;
+  a.b_offset = prob->b_offset;
   a.B = prob->B;
   a.R = prob->R;
   a.j = j;

@@ -30,6 +30,7 @@ WsPtrs ws_pointers(void* ws, const WsLayout& L);
 
 struct MaskArgs {
   uint64_t seed;
+  int32_t b_offset;   // global index of sequence 0 in the Philox counters
   int32_t B, R, j, n_t, t_mode;
   float* t_out;       // may be null
   uint8_t* mask_out;  // may be null

@@ -165,6 +165,7 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   }
   MaskArgs a;
   a.seed = prob->seed;
+  a.b_offset = prob->b_offset;
   a.B = prob->B;
   a.R = prob->R;
   a.j = j;

@@ -51,10 +51,11 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
     if (e < nblk) {
       b = (int32_t)(e / Q);
       q = (int32_t)(e % Q);
-      const PhiloxOut ot = philox4x64_10(0, (uint64_t)b, (uint64_t)a.j, kStreamT, a.seed, 0);
+      const uint64_t bg = (uint64_t)b + (uint64_t)a.b_offset;   // global sequence index
+      const PhiloxOut ot = philox4x64_10(0, bg, (uint64_t)a.j, kStreamT, a.seed, 0);
       const uint64_t u = ot.w[0] >> kU24Shift;
       const uint64_t T = (a.t_mode == 1) ? ((uint64_t)a.j << 24) + u + 1 : u + 1;
-      const PhiloxOut om = philox4x64_10((uint64_t)q, (uint64_t)b, (uint64_t)a.j, kStreamMask, a.seed, 0);
+      const PhiloxOut om = philox4x64_10((uint64_t)q, bg, (uint64_t)a.j, kStreamMask, a.seed, 0);
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const int32_t i = 4 * q + k;

@@ -29,12 +29,12 @@ def oracle_advantages(wl, inp):
     return O.group_advantage(to64(inp["rewards"]), wl.G)
 
 
-def oracle_run(wl, inp, loss_scale=None):
+def oracle_run(wl, inp, loss_scale=None, b_offset=0):
     """Algorithm 1 inner loops in fp64: draws, l_self, l_old = l_self + eps, bound, grads."""
     X, W, Y = to64(inp["X"]), to64(inp["W"]), to64(inp["Y"])
     ls = 1.0 / wl.G if loss_scale is None else loss_scale
     A = oracle_advantages(wl, inp)
-    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode)
+    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode, b_offset)
     ell_self = O.elbo_all(X, W, Y, wl.P, ts, masks)
     ell_old = ell_self + to64(inp["eps"])
     out = O.bgpo_step(X, W, Y, wl.P, A, ell_old, ts, masks, ls)
@@ -42,7 +42,7 @@ def oracle_run(wl, inp, loss_scale=None):
     return out
 
 
-def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None):
+def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
@@ -51,7 +51,7 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None):
     import torch
     import paper_2510_11683_gb300 as bg
 
-    prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale)
+    prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     B, n_t = wl.B, wl.n_t

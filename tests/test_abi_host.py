@@ -75,10 +75,12 @@ def test_validation_rejects_bad_problems(L, bg, kw, status):
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
 
 
-def test_validation_rejects_flags_and_nonfinite_scale(L, bg):
+def test_validation_rejects_bad_offset_and_nonfinite_scale(L, bg):
     p = _prob(bg)
-    p.flags = 1
+    p.b_offset = -1
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    p.b_offset = (1 << 31) - 1
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 2
     p = _prob(bg, loss_scale=float("nan"))
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
     assert L.bgpo_validate_problem(None) == 1

@@ -274,3 +274,27 @@ def test_trace_records_every_kernel(bg):
                      "bound_coeffs", "lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
     assert all(ms >= 0 for _, ms in tr.records())
     tr.close()
+
+
+def test_sequence_shards_reproduce_the_full_batch(bg):
+    """Data-parallel decomposition on one device: two shards with b_offset give
+    the whole batch's draws and l, and their dW sum to the whole batch's dW."""
+    import torch
+    wl = CONFIGS["ragged"].with_(B=6, G=3)
+    inp = make_inputs(wl, device="cuda")
+    full = gpu_run(wl, inp)
+    half = wl.with_(B=3)
+    parts = []
+    for k in range(2):
+        sl = slice(3 * k, 3 * k + 3)
+        sub = {"X": inp["X"][sl].contiguous(), "W": inp["W"], "Y": inp["Y"][sl].contiguous(),
+               "A": None, "rewards": inp["rewards"][sl].contiguous(),
+               "eps": inp["eps"][sl].contiguous()}
+        parts.append(gpu_run(half, sub, b_offset=3 * k))
+    assert torch.equal(torch.cat([p["masks"] for p in parts], dim=1), full["masks"])
+    ell = torch.cat([p["ell"] for p in parts])
+    assert torch.allclose(ell, full["ell"], rtol=1e-6, atol=1e-6)
+    dW = parts[0]["dW"] + parts[1]["dW"]
+    assert normwise(to64(dW), to64(full["dW"])) <= 1e-5
+    dX = torch.cat([p["dX"] for p in parts])
+    assert normwise(to64(dX), to64(full["dX"])) <= 1e-5

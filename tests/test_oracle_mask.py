@@ -73,3 +73,13 @@ def test_masks_are_a_pure_function_of_seed_b_j():
 def test_different_sequences_draw_independently():
     T, D, t, mask = O.sample_t_mask(8, 32, 64, 0, 1, 0)
     assert len(set(T.tolist())) == 32
+
+
+def test_shard_draws_match_the_full_batch():
+    # a data-parallel shard [b0, b0 + B) draws what the whole batch draws there
+    for t_mode in (0, 1):
+        Tf, Df, tf, mf = O.sample_t_mask(13, 12, 40, 3, 5, t_mode)
+        for b0, nb in ((0, 5), (5, 7), (11, 1)):
+            T, D, t, m = O.sample_t_mask(13, nb, 40, 3, 5, t_mode, b_offset=b0)
+            assert D == Df and (T == Tf[b0:b0 + nb]).all()
+            assert np.array_equal(m, mf[b0:b0 + nb])
