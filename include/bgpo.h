@@ -243,6 +243,16 @@ bgpo_status bgpo_get_device_error(const void* ws, size_t ws_bytes, int32_t* code
 /* Clears the device error word (asynchronous on `stream`). */
 bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * Failure-detection self-test: one warp waits, with the bounded wait every
+ * kernel of this library uses, on a barrier that nothing arrives at. After
+ * timeout_us (1 .. 1,000,000) the wait gives up and the kernel records
+ * BGPO_ERR_TIMEOUT in the workspace's device error word; the CUDA context stays
+ * usable. ws: a workspace (only its error word is touched).
+ */
+bgpo_status bgpo_selftest_bounded_wait(void* ws, size_t ws_bytes, uint32_t timeout_us,
+                                       void* stream);
+
 /* ---- per-kernel timing (host objects holding CUDA events) ---------------- */
 
 /* Creates a trace that can hold `capacity` kernel launches; NULL on failure. */

@@ -150,6 +150,14 @@ def clear_device_error(ws, stream=None):
     _lib.check("bgpo_clear_device_error", st)
 
 
+def selftest_bounded_wait(ws, timeout_us=2000, stream=None):
+    """Launches the bounded-wait self-test; read the result with get_device_error."""
+    torch = _torch()
+    st = _lib.lib().bgpo_selftest_bounded_wait(_ptr(ws, torch.uint8, "ws"), ws.numel(),
+                                               timeout_us, _stream(stream))
+    _lib.check("bgpo_selftest_bounded_wait", st)
+
+
 def kernel_name(kid):
     return _lib.lib().bgpo_kernel_name(kid).decode()
 

@@ -47,6 +47,7 @@ SIGNATURES = {
     "bgpo_get_device_error": (c_int32, [c_void_p, c_size_t, ctypes.POINTER(c_int32),
                                         ctypes.POINTER(c_int32), c_void_p]),
     "bgpo_clear_device_error": (c_int32, [c_void_p, c_size_t, c_void_p]),
+    "bgpo_selftest_bounded_wait": (c_int32, [c_void_p, c_size_t, ctypes.c_uint32, c_void_p]),
     "bgpo_trace_create": (c_void_p, [c_int32]),
     "bgpo_trace_destroy": (None, [c_void_p]),
     "bgpo_trace_reset": (None, [c_void_p]),

@@ -355,6 +355,19 @@ bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream) {
   return from_cuda(cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), static_cast<cudaStream_t>(stream)));
 }
 
+bgpo_status bgpo_selftest_bounded_wait(void* ws, size_t ws_bytes, uint32_t timeout_us,
+                                       void* stream) {
+  if (!ws) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
+  if (ws_bytes < 64) return BGPO_ERR_WORKSPACE_TOO_SMALL;
+  if (timeout_us == 0 || timeout_us > 1000000u) return BGPO_ERR_INVALID_ARG;
+  int sms = 0;
+  bgpo_status st = device_sms(&sms);
+  if (st != BGPO_OK) return st;
+  return from_cuda(launch_selftest_wait(static_cast<int32_t*>(ws), (uint64_t)timeout_us * 1000ull,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
 bgpo_trace* bgpo_trace_create(int32_t capacity) {
   if (capacity <= 0) return nullptr;
   bgpo_trace* t = static_cast<bgpo_trace*>(calloc(1, sizeof(bgpo_trace)));
@@ -407,7 +420,7 @@ const char* bgpo_kernel_name(int32_t id) {
   static const char* names[KID_COUNT] = {
       "mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
       "bound_coeffs", "lmhead_dz",   "dx_gemm",        "dx_reduce",   "dw_gemm",
-      "group_advantage"};
+      "group_advantage", "selftest_wait"};
   return (id >= 0 && id < KID_COUNT) ? names[id] : "?";
 }
 

@@ -67,18 +67,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Waits until the phase with parity `parity` of barrier `bar` has completed.
 // Returns false (without waiting further) when *abort becomes non-zero or the
-// wait runs out of time or polls.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+// wait runs out of time (timeout_ns) or polls.
+__device__ __forceinline__ bool mbar_wait_timeout(uint32_t bar, uint32_t parity,
+                                                  volatile int* abort, uint64_t timeout_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t poll = 1; poll < kWaitMaxPolls; ++poll) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((poll & 63u) == 0) {
       if (*abort) return false;
-      if (globaltimer_ns() - t0 > kWaitTimeoutNs) return false;
+      if (globaltimer_ns() - t0 > timeout_ns) return false;
     }
   }
   return false;
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+  return mbar_wait_timeout(bar, parity, abort, kWaitTimeoutNs);
 }
 
 // ---- TMA tensor loads (global -> shared, completion on an mbarrier) -------------

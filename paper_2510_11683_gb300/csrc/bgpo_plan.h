@@ -49,7 +49,8 @@ enum KernelId : int32_t {
   KID_DX_REDUCE = 8,
   KID_DW_GEMM = 9,
   KID_GROUP_ADV = 10,
-  KID_COUNT = 11
+  KID_SELFTEST_WAIT = 11,
+  KID_COUNT = 12
 };
 
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

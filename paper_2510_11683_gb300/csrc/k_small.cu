@@ -260,7 +260,32 @@ __global__ void k_group_advantage(int32_t B, int32_t G, const float* __restrict_
   for (int k = 0; k < G; ++k) A[grp * G + k] = sd > 0.f ? (x[k] - mean) / sd : 0.f;
 }
 
+// ---------------------------------------------------------------------------
+// Self-test of the bounded waits every kernel here uses: one warp waits on an
+// mbarrier that nothing arrives at; the wait must give up after timeout_ns and
+// record BGPO_ERR_TIMEOUT in the error word.
+// ---------------------------------------------------------------------------
+__global__ void k_selftest_wait(int32_t* err, uint64_t timeout_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  const uint32_t b = smem_addr(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(b, 1);
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncwarp();
+  const bool done = mbar_wait_timeout(b, 0, &abort_flag, timeout_ns);
+  if (!__all_sync(0xffffffffu, done) && threadIdx.x == 0)
+    set_device_error(err, 8 /* BGPO_ERR_TIMEOUT */, KID_SELFTEST_WAIT * 16);
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_wait(int32_t* err, uint64_t timeout_ns, cudaStream_t s) {
+  k_selftest_wait<<<1, 32, 0, s>>>(err, timeout_ns);
+  return cudaGetLastError();
+}
 
 WsPtrs ws_pointers(void* ws, const WsLayout& L) {
   char* base = static_cast<char*>(ws);

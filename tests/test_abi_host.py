@@ -38,7 +38,7 @@ def _declared_functions():
 def test_every_declared_symbol_is_exported(L):
     from paper_2510_11683_gb300 import _lib
     names = _declared_functions()
-    assert len(names) == len(_lib.SIGNATURES) == 18
+    assert len(names) == len(_lib.SIGNATURES) == 19
     for n in names:
         assert hasattr(L, n), n
         assert n in _lib.SIGNATURES, f"binding lacks {n}"
@@ -170,3 +170,10 @@ def test_binding_rejects_cpu_tensors(bg):
     p = _prob(bg)
     with pytest.raises(ValueError):
         bg.sample_mask(p, 0, torch.zeros(16, dtype=torch.uint8))
+
+
+def test_selftest_rejects_bad_arguments(L):
+    assert L.bgpo_selftest_bounded_wait(None, 1024, 100, None) == 1
+    assert L.bgpo_selftest_bounded_wait(FAKE + 8, 1024, 100, None) == 3
+    assert L.bgpo_selftest_bounded_wait(FAKE, 1024, 0, None) == 1
+    assert L.bgpo_selftest_bounded_wait(FAKE, 1024, 2000000, None) == 1

@@ -298,3 +298,24 @@ def test_sequence_shards_reproduce_the_full_batch(bg):
     assert normwise(to64(dW), to64(full["dW"])) <= 1e-5
     dX = torch.cat([p["dX"] for p in parts])
     assert normwise(to64(dX), to64(full["dX"])) <= 1e-5
+
+
+def test_bounded_wait_times_out_and_context_survives(bg):
+    """Failure detection on the device: a wait on a barrier nothing arrives at
+    gives up after its limit, the error word says BGPO_ERR_TIMEOUT, and the
+    next call on the same context works."""
+    import torch
+    wl, inp = _inputs("tiny")
+    p = bg.problem_from(wl)
+    ws = bg.alloc_workspace(p)
+    bg.clear_device_error(ws)
+    bg.selftest_bounded_wait(ws, timeout_us=5000)
+    code, where = bg.get_device_error(ws)
+    assert code == 8 and where == 11 * 16
+    bg.clear_device_error(ws)
+    ell = torch.empty(wl.B, device="cuda")
+    bg.sample_mask(p, 0, ws)
+    bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
+    torch.cuda.synchronize()
+    assert bg.get_device_error(ws) == (0, 0)
+    assert torch.isfinite(ell).all()
