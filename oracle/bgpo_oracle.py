@@ -194,6 +194,25 @@ def vrpo_ratio(ell, ell_old, A):
     return np.exp(ell.mean(axis=1) - ell_old.mean(axis=1)) * np.asarray(A, dtype=np.float64)
 
 
+def vrpo_coeffs(ell, ell_old, A, loss_scale):
+    """R_hat (Eq. 7) and dL/dl_{b,j} for L = -loss_scale * sum_b R_hat_b.
+
+    With B_hat the mean over the n_t samples (Eq. 5), dR_hat/dl_{b,j} =
+    e^{mean_j d_{b,j}} A_b / n_t for every j (Sec. 3.2). ell, ell_old [B, n_t];
+    returns (R_hat [B], coef [B]).
+    """
+    ell = np.asarray(ell, dtype=np.float64)
+    ell_old = np.asarray(ell_old, dtype=np.float64)
+    A = np.asarray(A, dtype=np.float64)
+    n_t = ell.shape[1]
+    e = np.exp(ell.mean(axis=1) - ell_old.mean(axis=1))
+    R = e * A
+    coef = -loss_scale * e * A / n_t
+    if not (np.all(np.isfinite(R)) and np.all(np.isfinite(coef))):
+        raise FloatingPointError("non-finite VRPO coefficient")
+    return R, coef
+
+
 def group_advantage(rewards, G):
     """Eq. 18: (r - mean_G r) / std_G r within consecutive groups of G responses.
 

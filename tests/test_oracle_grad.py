@@ -112,3 +112,30 @@ def test_linearity_accumulation_equals_one_shot():
         dW += gw
     assert np.allclose(dW, out["dW"], rtol=1e-12, atol=1e-14)
     assert np.allclose(dX, out["dX"], rtol=1e-12, atol=1e-14)
+
+
+def test_vrpo_coefficients_give_the_eq7_gradient_off_policy():
+    # the gradient of Eq. 7 assembled from per-sample coefficients, checked by
+    # central differences of the VRPO loss itself
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=7, n_t=4)
+    ell = O.elbo_all(X, W, Y, P, ts, masks)
+    R, coef = O.vrpo_coeffs(ell, ell_old, A, 0.5)
+    assert np.allclose(R, O.vrpo_ratio(ell, ell_old, A), rtol=1e-14)
+    dX = np.zeros((X.shape[0], masks.shape[2], X.shape[2]))
+    dW = np.zeros_like(W)
+    for j in range(len(ts)):
+        gx, gw = O.elbo_term_grads(X, W, Y, P, masks[j], ts[j], coef)
+        dX += gx
+        dW += gw
+    f = lambda X_, W_: O.vrpo_loss(X_, W_, Y, P, A, ell_old, ts, masks, 0.5)
+    _fd_check(f, X, W, dX, dW, P, seed=7)
+
+
+def test_vrpo_and_bgpo_coefficients_agree_on_policy():
+    # Sec. 3.2: with d = 0 both objectives weight every sample by -loss_scale A / n_t
+    rng = np.random.default_rng(8)
+    ell = rng.standard_normal((9, 5)) * 40
+    A = rng.standard_normal(9)
+    _, cv = O.vrpo_coeffs(ell, ell, A, 0.25)
+    _, _, cb = O.bound_coeffs(ell, ell, A[:, None], 5, 0.25)
+    assert np.allclose(cb, cv[:, None], rtol=1e-15, atol=0)
