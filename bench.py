@@ -453,48 +453,75 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev):
 
 
 def nt_sweep(bg, dev):
-    """Time and peak memory of one step vs n_t (8 x (256 + 512), LLaDA-8B head)."""
+    """Time and peak memory of one step vs n_t (8 x (256 + 512), LLaDA-8B head) for
+    BGPO and for the ELBO-based objective it bounds (VRPO, Eq. 7), whose weights
+    need every sample's l first: "vrpo_retain" keeps one workspace per sample
+    (memory grows with n_t), "vrpo_recompute" runs each sample's forward twice."""
     import torch
     from synth import CONFIGS, SWEEP_NT, make_inputs
     base = CONFIGS["llada8b_sweep"]
     inp0 = make_inputs(base.with_(n_t=max(SWEEP_NT)))
+    X, W, Y = inp0["X"].to(dev), inp0["W"].to(dev), inp0["Y"].to(dev)
+    rewards = inp0["rewards"].to(dev)
     res = []
     for n_t in SWEEP_NT:
         wl = base.with_(n_t=n_t)
-        torch.cuda.empty_cache()
-        torch.cuda.reset_peak_memory_stats(dev)
-        X, W, Y = inp0["X"].to(dev), inp0["W"].to(dev), inp0["Y"].to(dev)
         prob = bg.problem_from(wl)
-        ws = bg.alloc_workspace(prob, dev)
         A = torch.empty(wl.B, dtype=torch.float32, device=dev)
-        bg.group_advantage(prob, inp0["rewards"].to(dev), A)
-        ell = torch.empty((n_t, wl.B), dtype=torch.float32, device=dev)
-        coef, g = torch.empty_like(ell), torch.empty_like(ell)
-        dX = torch.zeros((wl.B, wl.R, wl.H), dtype=torch.float32, device=dev)
-        dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+        bg.group_advantage(prob, rewards, A)
         rows = 0
-
-        def run():
-            for j in range(n_t):
-                bg.sample_mask(prob, j, ws)
-                bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
-                bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
-                bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
-        run()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        run()
-        e1.record()
-        torch.cuda.synchronize()
         m = torch.empty((wl.B, wl.R), dtype=torch.uint8, device=dev)
+        ws0 = bg.alloc_workspace(prob, dev)
         for j in range(n_t):
-            bg.sample_mask(prob, j, ws, None, m)
+            bg.sample_mask(prob, j, ws0, None, m)
             rows += int(m.sum().item())
-        res.append({"n_t": n_t, "ms": e0.elapsed_time(e1), "masked_rows": rows,
-                    "tokens_per_s": rows / (e0.elapsed_time(e1) / 1e3),
-                    "peak_bytes": torch.cuda.max_memory_allocated(dev)})
-        del X, W, Y, ws, dX, dW
+        del ws0
+        point = {"n_t": n_t, "masked_rows": rows}
+        for method in ("bgpo", "vrpo_retain", "vrpo_recompute"):
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+            torch.cuda.reset_peak_memory_stats(dev)
+            n_ws = n_t if method == "vrpo_retain" else 1
+            wss = [bg.alloc_workspace(prob, dev) for _ in range(n_ws)]
+            ell = torch.empty((n_t, wl.B), dtype=torch.float32, device=dev)
+            coef, g = torch.empty_like(ell), torch.empty_like(ell)
+            cv = torch.empty(wl.B, dtype=torch.float32, device=dev)
+            tmp = torch.empty(wl.B, dtype=torch.float32, device=dev)
+            dX = torch.zeros((wl.B, wl.R, wl.H), dtype=torch.float32, device=dev)
+            dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+
+            def run():
+                if method == "bgpo":
+                    ws = wss[0]
+                    for j in range(n_t):
+                        bg.sample_mask(prob, j, ws)
+                        bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+                        bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
+                        bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
+                    return
+                for j in range(n_t):
+                    ws = wss[j % n_ws]
+                    bg.sample_mask(prob, j, ws)
+                    bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+                bg.vrpo_coeffs(prob, ell, ell, A, cv, None, wss[0])
+                for j in range(n_t):
+                    ws = wss[j % n_ws]
+                    if method == "vrpo_recompute":
+                        bg.sample_mask(prob, j, ws)
+                        bg.elbo_fwd(prob, j, X, W, Y, ws, tmp)
+                    bg.elbo_bwd_accumulate(prob, j, X, W, Y, cv, ws, dX, dW)
+            run()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            run()
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            point[method] = {"ms": ms, "tokens_per_s": rows / (ms / 1e3),
+                             "peak_bytes": torch.cuda.max_memory_allocated(dev)}
+            del wss, dX, dW
+        res.append(point)
     return res
 
 

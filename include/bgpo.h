@@ -15,7 +15,8 @@
  *                             accumulation; Linearity, Sec. 3), so memory does
  *                             not grow with n_t
  *
- * plus bgpo_group_advantage (Eq. 18).
+ * plus bgpo_group_advantage (Eq. 18) and, for comparison, the coefficients of
+ * the ELBO-based objective the bound replaces (bgpo_vrpo_coeffs, Eq. 7).
  *
  * Conventions shared by every call
  * --------------------------------
@@ -179,6 +180,24 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
 bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* ell,
                               const float* ell_old, const float* A, float* coef_out, float* g_out,
                               void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Coefficients of the ELBO-based objective BGPO bounds (VRPO, Eq. 7), for
+ * comparison with the bound: with B_hat the mean over the n_t samples (Eq. 5),
+ *   R_hat = e^{mean_j (l_{b,j} - l_old_{b,j})} A_b
+ *   coef  = dL/dl_{b,j} = -loss_scale * A_b * e^{mean_j d_{b,j}} / n_t  (every j)
+ * Unlike bgpo_bound_coeffs it needs all n_t samples' l before any backward
+ * pass: the caller either keeps every sample's workspace (memory grows with
+ * n_t) or runs each sample's forward twice. Feed coef to
+ * bgpo_elbo_bwd_accumulate for each j. On-policy (d = 0) it equals the
+ * bound's coefficient (Equivalence, Sec. 3.2).
+ *   ell, ell_old  device float [n_t, B] (row j = sample j);  A device float [B]
+ *   coef_out      device float [B];  R_out device float [B] or NULL
+ * A non-finite value sets the device error word to BGPO_ERR_NONFINITE.
+ */
+bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const float* ell_old,
+                             const float* A, float* coef_out, float* R_out, void* ws,
+                             size_t ws_bytes, void* stream);
 
 /*
  * Backward pass of L_j = sum_b coef_b * l_{b,j}, accumulated (Algorithm 1,

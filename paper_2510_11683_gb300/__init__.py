@@ -114,6 +114,17 @@ def bound_coeffs(prob, j, ell, ell_old, A, coef_out, g_out, ws, stream=None):
     _lib.check("bgpo_bound_coeffs", st)
 
 
+def vrpo_coeffs(prob, ell, ell_old, A, coef_out, R_out, ws, stream=None):
+    """Eq. 7 coefficients from all n_t samples' l ([n_t, B] tensors)."""
+    torch = _torch()
+    f32 = torch.float32
+    st = _lib.lib().bgpo_vrpo_coeffs(
+        ctypes.byref(prob), _ptr(ell, f32, "ell"), _ptr(ell_old, f32, "ell_old"),
+        _ptr(A, f32, "A"), _ptr(coef_out, f32, "coef_out"), _ptr(R_out, f32, "R_out"),
+        _ptr(ws, torch.uint8, "ws"), ws.numel(), _stream(stream))
+    _lib.check("bgpo_vrpo_coeffs", st)
+
+
 def elbo_bwd_accumulate(prob, j, X, W, Y, coef, ws, dX, dW, stream=None):
     torch = _torch()
     f32 = torch.float32

@@ -38,6 +38,8 @@ SIGNATURES = {
                                 c_void_p, c_size_t, c_void_p, c_void_p]),
     "bgpo_bound_coeffs": (c_int32, [ctypes.POINTER(BgpoProblem), c_int32, c_void_p, c_void_p,
                                     c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "bgpo_vrpo_coeffs": (c_int32, [ctypes.POINTER(BgpoProblem), c_void_p, c_void_p, c_void_p,
+                                   c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "bgpo_elbo_bwd_accumulate": (c_int32, [ctypes.POINTER(BgpoProblem), c_int32, c_void_p, c_void_p,
                                            c_void_p, c_void_p, c_void_p, c_size_t, c_void_p,
                                            c_void_p, c_void_p]),

@@ -257,6 +257,26 @@ bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* 
                                        coef_out, g_out, w, s));
 }
 
+bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const float* ell_old,
+                             const float* A, float* coef_out, float* R_out, void* ws,
+                             size_t ws_bytes, void* stream) {
+  bgpo_status st = check_problem(prob);
+  if (st != BGPO_OK) return st;
+  if (!ell || !ell_old || !A || !coef_out) return BGPO_ERR_INVALID_ARG;
+  if (!aligned(ell, 4) || !aligned(ell_old, 4) || !aligned(A, 4) || !aligned(coef_out, 4) ||
+      (R_out && !aligned(R_out, 4)))
+    return BGPO_ERR_ALIGNMENT;
+  WsLayout L;
+  if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
+  int sms = 0;
+  if ((st = device_sms(&sms)) != BGPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const WsPtrs w = ws_pointers(ws, L);
+  TraceScope ts(prob->trace, KID_VRPO_COEFFS, s);
+  return from_cuda(launch_vrpo_coeffs(prob->B, prob->n_t, prob->loss_scale, ell, ell_old, A,
+                                      coef_out, R_out, w, s));
+}
+
 bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
                                      const void* W, const int32_t* Y, const float* coef, void* ws,
                                      size_t ws_bytes, float* dX, float* dW, void* stream) {
@@ -420,7 +440,7 @@ const char* bgpo_kernel_name(int32_t id) {
   static const char* names[KID_COUNT] = {
       "mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
       "bound_coeffs", "lmhead_dz",   "dx_gemm",        "dx_reduce",   "dw_gemm",
-      "group_advantage", "selftest_wait"};
+      "group_advantage", "selftest_wait", "vrpo_coeffs"};
   return (id >= 0 && id < KID_COUNT) ? names[id] : "?";
 }
 

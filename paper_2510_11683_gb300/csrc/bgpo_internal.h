@@ -49,6 +49,9 @@ cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_pairs, const 
                              float* dX, cudaStream_t s);
 cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
                                    cudaStream_t s);
+cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
+                               const float* ell_old, const float* A, float* coef_out, float* R_out,
+                               const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_selftest_wait(int32_t* err, uint64_t timeout_ns, cudaStream_t s);
 
 // The four tcgen05 GEMMs of the path.

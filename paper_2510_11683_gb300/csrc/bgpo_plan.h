@@ -50,7 +50,8 @@ enum KernelId : int32_t {
   KID_DW_GEMM = 9,
   KID_GROUP_ADV = 10,
   KID_SELFTEST_WAIT = 11,
-  KID_COUNT = 12
+  KID_VRPO_COEFFS = 12,
+  KID_COUNT = 13
 };
 
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

@@ -219,6 +219,27 @@ __global__ void k_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const f
 }
 
 // ---------------------------------------------------------------------------
+// VRPO (Eq. 7): R_hat = e^{mean_j (l - l_old)} A and dL/dl_{b,j} =
+// -loss_scale A e^{mean_j d} / n_t for every j (Sec. 3.2). l, l_old [n_t, B].
+// ---------------------------------------------------------------------------
+__global__ void k_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* __restrict__ ell,
+                              const float* __restrict__ ell_old, const float* __restrict__ A,
+                              float* coef_out, float* R_out, int32_t* err) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  float sum_d = 0.f;
+  for (int j = 0; j < n_t; ++j) sum_d += ell[(int64_t)j * B + b] - ell_old[(int64_t)j * B + b];
+  const float inv_nt = 1.f / (float)n_t;
+  const float e = expf(sum_d * inv_nt);
+  const float a = A[b];
+  const float R = e * a;
+  const float coef = -loss_scale * a * e * inv_nt;
+  coef_out[b] = coef;
+  if (R_out) R_out[b] = R;
+  if (!isfinite(R) || !isfinite(coef)) set_device_error(err, kStatusNonfinite, KID_VRPO_COEFFS * 16);
+}
+
+// ---------------------------------------------------------------------------
 // dX[b, i, :] += sum_s partial_s[r, :] over the split-K partials of the dX GEMM
 // (fixed split order; rows are unique within a sample, so no atomics).
 // ---------------------------------------------------------------------------
@@ -336,6 +357,14 @@ cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const 
                                 float* g_out, const WsPtrs& w, cudaStream_t s) {
   k_bound_coeffs<<<(unsigned)ceil_div(B, 256), 256, 0, s>>>(B, n_t, loss_scale, ell, ell_old, A,
                                                             coef_out, g_out, w.err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
+                               const float* ell_old, const float* A, float* coef_out, float* R_out,
+                               const WsPtrs& w, cudaStream_t s) {
+  k_vrpo_coeffs<<<(unsigned)ceil_div(B, 256), 256, 0, s>>>(B, n_t, loss_scale, ell, ell_old, A,
+                                                           coef_out, R_out, w.err);
   return cudaGetLastError();
 }
 

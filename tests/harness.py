@@ -95,3 +95,62 @@ def normwise(got, ref):
     ref = np.asarray(ref, dtype=np.float64)
     den = np.linalg.norm(ref)
     return np.linalg.norm(got - ref) / (den if den > 0 else 1.0)
+
+
+def oracle_run_vrpo(wl, inp, loss_scale=None):
+    """The ELBO-based objective of Eq. 7 in fp64: R_hat and its accumulated gradients."""
+    X, W, Y = to64(inp["X"]), to64(inp["W"]), to64(inp["Y"])
+    ls = 1.0 / wl.G if loss_scale is None else loss_scale
+    A = oracle_advantages(wl, inp)
+    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode)
+    ell = O.elbo_all(X, W, Y, wl.P, ts, masks)
+    ell_old = ell + to64(inp["eps"])
+    R, coef = O.vrpo_coeffs(ell, ell_old, A, ls)
+    dX = np.zeros((wl.B, wl.R, wl.H))
+    dW = np.zeros((wl.V, wl.H))
+    for j in range(wl.n_t):
+        gx, gw = O.elbo_term_grads(X, W, Y, wl.P, masks[j], ts[j], coef)
+        dX += gx
+        dW += gw
+    return dict(ell=ell, R=R, coef=coef, dX=dX, dW=dW)
+
+
+def gpu_run_vrpo(wl, inp, strategy, dev="cuda"):
+    """Eq. 7 through the C ABI. strategy "retain": one workspace per MC sample
+    (forward state kept for all n_t samples); "recompute": one workspace, each
+    sample's forward run again before its backward."""
+    import torch
+    import paper_2510_11683_gb300 as bg
+
+    prob = bg.problem_from(wl)
+    B, n_t = wl.B, wl.n_t
+    X, W, Y = inp["X"], inp["W"], inp["Y"]
+    A = torch.empty(B, dtype=torch.float32, device=dev)
+    if inp["A"] is not None:
+        A.copy_(inp["A"])
+    else:
+        bg.group_advantage(prob, inp["rewards"], A)
+    n_ws = n_t if strategy == "retain" else 1
+    wss = [bg.alloc_workspace(prob, dev) for _ in range(n_ws)]
+    for ws in wss:
+        bg.clear_device_error(ws)
+    ell = torch.empty((n_t, B), dtype=torch.float32, device=dev)
+    for j in range(n_t):
+        ws = wss[j % n_ws]
+        bg.sample_mask(prob, j, ws)
+        bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+    ell_old = (ell + inp["eps"].T).contiguous()
+    coef = torch.empty(B, dtype=torch.float32, device=dev)
+    R = torch.empty(B, dtype=torch.float32, device=dev)
+    bg.vrpo_coeffs(prob, ell, ell_old, A, coef, R, wss[0])
+    dX = torch.zeros((B, wl.R, wl.H), dtype=torch.float32, device=dev)
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+    tmp = torch.empty(B, dtype=torch.float32, device=dev)
+    for j in range(n_t):
+        ws = wss[j % n_ws]
+        if strategy != "retain":
+            bg.sample_mask(prob, j, ws)
+            bg.elbo_fwd(prob, j, X, W, Y, ws, tmp)
+        bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef, ws, dX, dW)
+    torch.cuda.synchronize()
+    return dict(ell=ell.T, R=R, coef=coef, dX=dX, dW=dW, ws=wss)

@@ -38,7 +38,7 @@ def _declared_functions():
 def test_every_declared_symbol_is_exported(L):
     from paper_2510_11683_gb300 import _lib
     names = _declared_functions()
-    assert len(names) == len(_lib.SIGNATURES) == 19
+    assert len(names) == len(_lib.SIGNATURES) == 20
     for n in names:
         assert hasattr(L, n), n
         assert n in _lib.SIGNATURES, f"binding lacks {n}"
