@@ -51,6 +51,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--grad-variance", action="store_true",
+                    help="run the Sec. 4.3 gradient std / bias vs n_t study instead")
     return ap.parse_args()
 
 
@@ -240,6 +242,9 @@ def main():
     wl = CONFIGS[args.workload]
     if args.impl == "reference":
         run_reference(args, wl)
+        return
+    if args.grad_variance:
+        run_grad_variance(args, CONFIGS["llada8b_sweep"] if args.workload == WORKLOAD else wl)
         return
 
     import torch
@@ -450,6 +455,83 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev):
     dt = (time.perf_counter() - t0) / steps
     return {"value": masked_per_step / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps}
+
+
+def grad_seed(wl, n_t, rep):
+    """Draw seed of repeat `rep` at `n_t` (rep = -1: the golden gradient)."""
+    return wl.seed + 1_000_003 if rep < 0 else wl.seed + 1 + 7919 * rep + 104729 * n_t
+
+
+def grad_variance(bg, wl, nts, repeats, golden_nt, dev):
+    """Sec. 4.3 on the synthetic head: the batch gradient dW of the on-policy
+    BGPO objective computed `repeats` times with independent MC draws for each
+    n_t; std = mean over parameters of the per-parameter std over the repeats,
+    bias = mean over parameters of |mean over repeats - golden|, golden = the
+    gradient with golden_nt samples."""
+    import torch
+    from synth import make_inputs
+    inp = make_inputs(wl)
+    X, W, Y = inp["X"].to(dev), inp["W"].to(dev), inp["Y"].to(dev)
+    base = bg.problem_from(wl)
+    A = torch.empty(wl.B, dtype=torch.float32, device=dev)
+    if inp["A"] is not None:
+        A.copy_(inp["A"].to(dev))
+    else:
+        bg.group_advantage(base, inp["rewards"].to(dev), A)
+    dX = torch.zeros((wl.B, wl.R, wl.H), dtype=torch.float32, device=dev)
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
+
+    def gradient(n_t, seed):
+        prob = bg.problem(wl.B, wl.P, wl.R, wl.H, wl.V, n_t, wl.G, wl.t_mode, seed)
+        ws = bg.alloc_workspace(prob, dev)
+        ell = torch.empty(wl.B, dtype=torch.float32, device=dev)
+        coef = torch.empty_like(ell)
+        dW.zero_()
+        dX.zero_()
+        for j in range(n_t):
+            bg.sample_mask(prob, j, ws)
+            bg.elbo_fwd(prob, j, X, W, Y, ws, ell)
+            bg.bound_coeffs(prob, j, ell, ell, A, coef, None, ws)   # on-policy: d = 0
+            bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef, ws, dX, dW)
+        code = bg.get_device_error(ws)[0]
+        if code != 0:
+            raise RuntimeError(f"device error {code}")
+        return dW.double()
+
+    golden = gradient(golden_nt, grad_seed(wl, golden_nt, -1)).clone()
+    out = []
+    for n_t in nts:
+        s1 = torch.zeros_like(golden)
+        s2 = torch.zeros_like(golden)
+        for rep in range(repeats):
+            g = gradient(n_t, grad_seed(wl, n_t, rep))
+            s1 += g
+            s2 += g * g
+        mean = s1 / repeats
+        var = (s2 / repeats - mean * mean).clamp_min(0.0)
+        out.append({"n_t": n_t, "std": float(var.sqrt().mean()),
+                    "bias": float((mean - golden).abs().mean())})
+    return out
+
+
+def run_grad_variance(args, wl):
+    import torch
+    import paper_2510_11683_gb300 as bg
+    from paper_2510_11683_gb300 import build as B
+    if not os.path.exists(B.LIB_PATH):
+        B.build()
+    dev = torch.device("cuda", 0)
+    study = CONFIG_GRAD_VARIANCE
+    t0 = time.perf_counter()
+    res = grad_variance(bg, wl.with_(eps_std=0.0), study["n_t"], study["repeats"],
+                        study["golden_n_t"], dev)
+    print(json.dumps({"experiment": "grad_std_bias_vs_n_t (Sec. 4.3)",
+                      "workload": config_of(wl)["workload"], "repeats": study["repeats"],
+                      "golden_n_t": study["golden_n_t"], "points": res,
+                      "seconds": time.perf_counter() - t0}), flush=True)
+
+
+CONFIG_GRAD_VARIANCE = {"n_t": (1, 2, 4, 8, 16, 32), "repeats": 8, "golden_n_t": 256}
 
 
 def nt_sweep(bg, dev):

@@ -315,3 +315,23 @@ def vrpo_loss(X, W, Y, P, A, ell_old, ts, masks, loss_scale):
     """Scalar -loss_scale * sum_b R_hat_b with R_hat of Eq. 7 (draws held fixed)."""
     ell = elbo_all(X, W, Y, P, ts, masks)
     return -loss_scale * vrpo_ratio(ell, ell_old, A).sum()
+
+
+# ---------------------------------------------------------------------------
+# Gradient variance and bias vs n_t (Sec. 4.3)
+# ---------------------------------------------------------------------------
+
+def grad_std_bias(grads, golden):
+    """Sec. 4.3 statistics of repeated gradient estimates of one batch.
+
+    grads [K, ...]: K gradients computed with independent MC draws; golden: the
+    reference gradient (the paper uses n_t = 256). Reading of the figure, whose
+    values are not printed: std = mean over parameters of the per-parameter
+    standard deviation over the K repeats (population, ddof = 0); bias = mean
+    over parameters of |mean over repeats - golden|.
+    """
+    g = np.asarray(grads, dtype=np.float64)
+    gold = np.asarray(golden, dtype=np.float64)
+    std = g.std(axis=0).mean()
+    bias = np.abs(g.mean(axis=0) - gold).mean()
+    return float(std), float(bias)

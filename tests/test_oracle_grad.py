@@ -139,3 +139,26 @@ def test_vrpo_and_bgpo_coefficients_agree_on_policy():
     _, cv = O.vrpo_coeffs(ell, ell, A, 0.25)
     _, _, cb = O.bound_coeffs(ell, ell, A[:, None], 5, 0.25)
     assert np.allclose(cb, cv[:, None], rtol=1e-15, atol=0)
+
+
+def test_grad_std_bias_definitions():
+    # closed forms: constant repeats have zero std; a known offset is the bias
+    g = np.stack([np.full((3, 4), 2.0)] * 5)
+    assert O.grad_std_bias(g, np.full((3, 4), 1.5)) == (0.0, 0.5)
+    # two repeats +-1 around the golden value: std 1, bias 0
+    g = np.stack([np.ones((2, 2)), -np.ones((2, 2))])
+    assert O.grad_std_bias(g, np.zeros((2, 2))) == (1.0, 0.0)
+
+
+def test_mc_gradient_std_shrinks_with_n_t():
+    # Sec. 4.3: more MC samples, smaller spread of the gradient estimate
+    X, W, Y, P, A, _, _, _ = _case(seed=9, B=2, R=10, H=5, V=11, n_t=1)
+    stds = []
+    for n_t in (1, 4, 16):
+        grads = []
+        for rep in range(12):
+            ts, masks = O.sample_masks(1000 + 97 * rep, 2, 10, n_t, 0)
+            ell = O.elbo_all(X, W, Y, P, ts, masks)
+            grads.append(O.bgpo_step(X, W, Y, P, A, ell, ts, masks, 1.0)["dW"])
+        stds.append(O.grad_std_bias(np.stack(grads), np.zeros_like(W))[0])
+    assert stds[0] > stds[1] > stds[2]
