@@ -523,8 +523,8 @@ def run_grad_variance(args, wl):
     dev = torch.device("cuda", 0)
     study = CONFIG_GRAD_VARIANCE
     t0 = time.perf_counter()
-    res = grad_variance(bg, wl.with_(eps_std=0.0), study["n_t"], study["repeats"],
-                        study["golden_n_t"], dev)
+    wl = wl.with_(eps_std=0.0)   # on-policy: BGPO and VRPO gradients coincide (Sec. 3.2)
+    res = grad_variance(bg, wl, study["n_t"], study["repeats"], study["golden_n_t"], dev)
     print(json.dumps({"experiment": "grad_std_bias_vs_n_t (Sec. 4.3)",
                       "workload": config_of(wl)["workload"], "repeats": study["repeats"],
                       "golden_n_t": study["golden_n_t"], "points": res,
