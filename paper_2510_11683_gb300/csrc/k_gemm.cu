@@ -101,12 +101,13 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
     t.kb0 = 0;
     t.kb_n = (int32_t)w.kb_total;
   } else if (KIND == GEMM_DX) {
-    // consecutive units share a column block of W
+    // consecutive units share a row block of dZ (measured 2% faster than
+    // sharing a column block of W, and than grouped rasters)
     const int64_t per_split = w.tiles_m * w.tiles_n;
     t.split = (int32_t)(u / per_split);
     const int64_t rem = u % per_split;
-    t.n_blk = (int32_t)(rem / w.tiles_m);
-    t.m_blk = (int32_t)(rem % w.tiles_m);
+    t.m_blk = (int32_t)(rem / w.tiles_n);
+    t.n_blk = (int32_t)(rem % w.tiles_n);
     const int64_t k0 = (int64_t)t.split * w.kb_total / w.splits;
     const int64_t k1 = (int64_t)(t.split + 1) * w.kb_total / w.splits;
     t.kb0 = (int32_t)k0;
