@@ -33,11 +33,14 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant kernel,
-# from the ncu capture summarised in profiles/ (scaled to this workload's masked
-# rows per launch). Valid only while the kernel source is unchanged.
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of dw_gemm, from the
+# ncu capture of all 16 launches of the llada8b_r512_b8 case summarised in
+# profiles/dw_gemm_traffic_llada8b_r512_b8.md: an affine fit in the launch's
+# masked rows M (the dW read-modify-write is fixed, dZ / Xm reads grow with M).
+# Valid only while the GEMM sources hash to `sha`.
 TRAFFIC = {
-    # kernel name: (bytes per masked row, sha256 of k_gemm.cu when captured)
+    "dw_gemm": {"fixed_bytes": 4.0237e9, "bytes_per_row": 350337.7,
+                "sha": "47e99795f0eabbd87d82483f9de73573a2a391cfcf76d0d24dd57da317f6085f"},
 }
 
 
@@ -232,8 +235,12 @@ def shard_of(wl, rank, world):
 
 
 def kernel_sha():
-    with open(os.path.join(ROOT, "paper_2510_11683_gb300", "csrc", "k_gemm.cu"), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()
+    """sha256 of the GEMM kernel sources (k_gemm.cu and the headers it inlines)."""
+    h = hashlib.sha256()
+    for name in ("k_gemm.cu", "bgpo_device.cuh", "bgpo_plan.h"):
+        with open(os.path.join(ROOT, "paper_2510_11683_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 def main():
@@ -351,8 +358,8 @@ def main():
     dom_avg_s = dom_ms / dom_launches / 1e3
     achieved = dom_flops_per_launch / dom_avg_s / 1e12
     traffic = None
-    if dom in TRAFFIC and TRAFFIC[dom][1] == kernel_sha():
-        traffic = TRAFFIC[dom][0] * masked_per_step / n_t
+    if dom in TRAFFIC and TRAFFIC[dom]["sha"] == kernel_sha():
+        traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * masked_per_step / n_t
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
