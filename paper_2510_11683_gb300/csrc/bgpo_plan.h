@@ -33,8 +33,6 @@ constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
 // 128-byte sub-tile (32 fp32 or 64 bf16 columns) for its TMA stores.
 constexpr uint32_t kEpiBufBytes = 32 * 128;
 constexpr uint32_t kEpiBytes = 4 * 2 * kEpiBufBytes;   // 32 KB
-constexpr uint32_t kGemmSmemBytes =
-    kStages * kStageBytes + kEpiBytes + 1024 /*barriers*/ + 1024 /*align*/;
 
 // ---- kernel ids (trace + device error "where") --------------------------------
 enum KernelId : int32_t {

@@ -122,6 +122,17 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
   return t;
 }
 
+// Shared-memory plan of one kind: the forward GEMM writes no tiles from its
+// epilogue and needs no staging space (a 7th stage in that space measured no
+// faster than 6).
+template <int KIND>
+struct SmemPlan {
+  static constexpr int stages = kStages;
+  static constexpr uint32_t epi_bytes = (KIND == GEMM_FWD) ? 0u : kEpiBytes;
+  static constexpr uint32_t bytes = stages * kStageBytes + epi_bytes + 1024 + 1024;
+  static_assert(bytes <= 232448, "shared memory per CTA");
+};
+
 template <int KIND>
 struct Majors {
   static constexpr bool a_mn = (KIND == GEMM_DW);
@@ -385,19 +396,20 @@ template <int KIND>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
            const __grid_constant__ CUtensorMap map_c, const GemmParams p) {
+  constexpr int kSt = SmemPlan<KIND>::stages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* s_a = smem;
-  uint8_t* s_b = smem + kStages * kTileABytes;
-  uint8_t* s_epi = s_b + kStages * kTileBBytes;   // 4 warps x 2 staging buffers
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_epi + kEpiBytes);
-  uint64_t* full = bars;                      // [kStages] TMA (both CTAs) -> MMA; even CTA's
-  uint64_t* empty = bars + kStages;           // [kStages] MMA -> TMA of each CTA
-  uint64_t* tfull = bars + 2 * kStages;       // [2] MMA -> epilogue of each CTA
-  uint64_t* tempty = bars + 2 * kStages + 2;  // [2] epilogues (both CTAs) -> MMA; even CTA's
-  uint64_t* done = bars + 2 * kStages + 4;    // MMA drain on abort
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 5);
+  uint8_t* s_b = smem + kSt * kTileABytes;
+  uint8_t* s_epi = s_b + kSt * kTileBBytes;   // 4 warps x 2 staging buffers (not GEMM_FWD)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_epi + SmemPlan<KIND>::epi_bytes);
+  uint64_t* full = bars;                      // [kSt] TMA (both CTAs) -> MMA; even CTA's
+  uint64_t* empty = bars + kSt;           // [kSt] MMA -> TMA of each CTA
+  uint64_t* tfull = bars + 2 * kSt;       // [2] MMA -> epilogue of each CTA
+  uint64_t* tempty = bars + 2 * kSt + 2;  // [2] epilogues (both CTAs) -> MMA; even CTA's
+  uint64_t* done = bars + 2 * kSt + 4;    // MMA drain on abort
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kSt + 5);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* never = reinterpret_cast<volatile int*>(tmem_slot + 2);
 
@@ -419,7 +431,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (pair >= wk.units) return;  // both CTAs of the pair, before any allocation
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kSt; ++s) {
       mbar_init(smem_addr(&full[s]), 1);    // the even CTA's arrive.expect_tx
       mbar_init(smem_addr(&empty[s]), 1);   // one multicast commit
     }
@@ -467,7 +479,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           load_stage<KIND>(p, &map_a, &map_b, smem_addr(s_a + stage * kTileABytes),
                            smem_addr(s_b + stage * kTileBBytes), cbar, t, kb, rank);
           issued = true;
-          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          if (++stage == kSt) { stage = 0; phase ^= 1u; }
         }
       }
       if (!ok) {
@@ -514,7 +526,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           issued = true;
           // frees this stage in both CTAs once these MMAs have read it
           umma_commit_pair(smem_addr(&empty[stage]), kBothCtas);
-          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          if (++stage == kSt) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
         umma_commit_pair(smem_addr(&tfull[acc]), kBothCtas);  // accumulators ready
@@ -574,10 +586,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 template <int KIND>
 cudaError_t launch_kind(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc,
                         const GemmParams& p, cudaStream_t s) {
+  constexpr uint32_t smem = SmemPlan<KIND>::bytes;
   cudaError_t e = cudaFuncSetAttribute(k_gemm<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kGemmSmemBytes);
+                                       (int)smem);
   if (e != cudaSuccess) return e;
-  k_gemm<KIND><<<2 * p.num_pairs, kThreads, kGemmSmemBytes, s>>>(ma, mb, mc, p);
+  k_gemm<KIND><<<2 * p.num_pairs, kThreads, smem, s>>>(ma, mb, mc, p);
   return cudaGetLastError();
 }
 
@@ -591,9 +604,9 @@ int gemm_num_pairs(int num_sms) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)num_sms, 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kGemmSmemBytes;
+    cfg.dynamicSmemBytes = SmemPlan<GEMM_DX>::bytes;
     if (cudaFuncSetAttribute(k_gemm<GEMM_DX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kGemmSmemBytes) == cudaSuccess &&
+                             (int)SmemPlan<GEMM_DX>::bytes) == cudaSuccess &&
         cudaOccupancyMaxActiveClusters(&clusters, k_gemm<GEMM_DX>, &cfg) == cudaSuccess &&
         clusters > 0)
       cached = clusters;
