@@ -69,11 +69,13 @@ def mask_bit(u24, T, D):
     return int(int(u24) * int(D) < int(T) * TWO24)
 
 
-def sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset=0):
+def sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset=0, resp_len=None):
     """Timesteps and response masks of MC sample j for B sequences.
 
     Sequence b of this batch has global index b_offset + b in the counters, so a
     shard of a larger batch draws what the whole batch draws for those rows.
+    resp_len [B] (optional): response b holds resp_len[b] <= R tokens; positions
+    i >= resp_len[b] are padding and never masked (the draws are unchanged).
     Returns (T [B] int64, D int, t [B] float64, mask [B, R] uint8). Prompt
     positions are never masked (Sec. 2.1), so only the R response positions
     appear here.
@@ -88,6 +90,8 @@ def sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset=0):
     words = philox4x64_10_array(q, bb, np.uint64(j), np.uint64(STREAM_MASK), seed, 0)
     u = np.stack(words, axis=-1).reshape(B, Q * 4)[:, :R] >> np.uint64(U24_SHIFT)
     mask = mask_bit(u, T.astype(np.uint64)[:, None], D)
+    if resp_len is not None:
+        mask = mask * (np.arange(R)[None, :] < np.asarray(resp_len)[:, None]).astype(np.uint8)
     t = T.astype(np.float64) / float(D)
     return T, D, t, mask
 
@@ -266,11 +270,11 @@ def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192):
 # Algorithm 1, inner loops: all n_t MC samples of one batch
 # ---------------------------------------------------------------------------
 
-def sample_masks(seed, B, R, n_t, t_mode, b_offset=0):
+def sample_masks(seed, B, R, n_t, t_mode, b_offset=0, resp_len=None):
     """(t [n_t, B], mask [n_t, B, R]) for every MC sample j."""
     ts, masks = [], []
     for j in range(n_t):
-        _, _, t, m = sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset)
+        _, _, t, m = sample_t_mask(seed, B, R, j, n_t, t_mode, b_offset, resp_len)
         ts.append(t)
         masks.append(m)
     return np.stack(ts), np.stack(masks)

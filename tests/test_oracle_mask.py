@@ -83,3 +83,35 @@ def test_shard_draws_match_the_full_batch():
             T, D, t, m = O.sample_t_mask(13, nb, 40, 3, 5, t_mode, b_offset=b0)
             assert D == Df and (T == Tf[b0:b0 + nb]).all()
             assert np.array_equal(m, mf[b0:b0 + nb])
+
+
+def test_padding_positions_are_never_masked():
+    # variable-length responses: positions at or past the length stay unmasked,
+    # the draws of the real positions are those of the full-length response
+    lens = np.array([37, 0, 12, 40])
+    T0, D0, t0, m0 = O.sample_t_mask(21, 4, 40, 2, 4, 0)
+    T, D, t, m = O.sample_t_mask(21, 4, 40, 2, 4, 0, resp_len=lens)
+    assert (T == T0).all() and np.array_equal(t, t0)
+    for b, n in enumerate(lens):
+        assert np.array_equal(m[b, :n], m0[b, :n]) and not m[b, n:].any()
+
+
+def test_brute_force_unbiased_with_padding():
+    # Eq. 3-4 over the real tokens only: E_mask[l] = sum_{i < len} log p(y^i)
+    import itertools
+    import torch
+    rng = np.random.default_rng(31)
+    R, n = 9, 6
+    X = rng.standard_normal((1, R, 5))
+    W = rng.standard_normal((7, 5))
+    Y = rng.integers(0, 7, size=(1, R))
+    z = torch.from_numpy(X[0, :n]) @ torch.from_numpy(W).T
+    exact = float(torch.log_softmax(z, 1).gather(1, torch.from_numpy(Y[0, :n]).long()[:, None]).sum())
+    t = 0.42
+    acc = 0.0
+    for bits in itertools.product((0, 1), repeat=n):
+        m = np.zeros((1, R), dtype=np.uint8)
+        m[0, :n] = bits
+        k = sum(bits)
+        acc += t ** k * (1 - t) ** (n - k) * O.elbo_term(X, W, Y, 0, m, np.array([t]))[0]
+    assert abs(acc - exact) < 1e-12 * abs(exact)
