@@ -94,6 +94,10 @@ typedef struct bgpo_trace bgpo_trace;
  *          shard holding sequences [b_offset, b_offset + B) of a larger batch
  *          draws exactly the t and masks the whole batch would draw for them.
  *   trace  optional bgpo_trace* (NULL = off)
+ *   resp_len  optional device int32 [B] (NULL = every response has R tokens):
+ *          response b holds resp_len[b] tokens (0 <= resp_len[b] <= R); positions
+ *          i >= resp_len[b] are padding and never masked (the draws of the other
+ *          positions are unchanged; values outside [0, R] are clamped)
  * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
  * bgpo_workspace_bytes).
  */
@@ -110,6 +114,7 @@ typedef struct bgpo_problem {
   float loss_scale;
   int32_t b_offset;
   bgpo_trace* trace;
+  const int32_t* resp_len;
 } bgpo_problem;
 
 /* ABI version of the loaded library (BGPO_ABI_VERSION). */
@@ -140,7 +145,8 @@ size_t bgpo_workspace_bytes(const bgpo_problem* prob);
  * stratified; u24 = top 24 bits of output word 0) and masks response position
  * i of sequence b iff u24_i * D < T * 2^24, where u24_i is the top 24 bits of
  * output word (i mod 4) of the block with counter (i / 4, b', j, 0). Prompt
- * positions are never masked. Compacts the masked positions into ascending
+ * positions, and response positions at or past resp_len[b], are never masked.
+ * Compacts the masked positions into ascending
  * (b, i) order inside the workspace.
  *   j         sample index, 0 <= j < n_t
  *   ws        device workspace (256-byte aligned), ws_bytes its size

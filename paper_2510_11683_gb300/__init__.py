@@ -26,24 +26,27 @@ def _torch():
 
 
 def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None,
-            b_offset=0):
+            b_offset=0, resp_len=None):
     """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1).
 
     b_offset: global index of the first sequence (a data-parallel shard of a
-    larger batch draws the same t and masks as the whole batch would)."""
+    larger batch draws the same t and masks as the whole batch would).
+    resp_len: optional int32 CUDA tensor [B] of real response lengths (padding
+    positions are never masked); the tensor must outlive the calls."""
     p = BgpoProblem()
     p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
     p.seed = seed
     p.loss_scale = (1.0 / G if G > 0 else 1.0) if loss_scale is None else loss_scale
     p.b_offset = b_offset
+    p.resp_len = _ptr(resp_len, _torch().int32, "resp_len") if resp_len is not None else None
     p.trace = trace.handle if isinstance(trace, Trace) else trace
     return p
 
 
-def problem_from(wl, trace=None, loss_scale=None, b_offset=0):
+def problem_from(wl, trace=None, loss_scale=None, b_offset=0, resp_len=None):
     """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
     return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
-                   loss_scale=loss_scale, trace=trace, b_offset=b_offset)
+                   loss_scale=loss_scale, trace=trace, b_offset=b_offset, resp_len=resp_len)
 
 
 def validate_problem(prob):
@@ -58,10 +61,13 @@ def workspace_bytes(prob):
 
 
 def alloc_workspace(prob, device="cuda"):
-    """A uint8 device tensor of workspace_bytes(prob) (256-byte aligned by torch)."""
+    """A uint8 device tensor of workspace_bytes(prob) (256-byte aligned by torch)
+    with a cleared device error word (the rest is scratch the calls overwrite)."""
     torch = _torch()
     ws = torch.empty(workspace_bytes(prob), dtype=torch.uint8, device=device)
     assert ws.data_ptr() % 256 == 0
+    with torch.cuda.device(ws.device):
+        clear_device_error(ws)
     return ws
 
 

@@ -22,7 +22,7 @@ class BgpoProblem(ctypes.Structure):
         ("B", c_int32), ("P", c_int32), ("R", c_int32), ("H", c_int32), ("V", c_int32),
         ("n_t", c_int32), ("G", c_int32), ("t_mode", c_int32),
         ("seed", ctypes.c_uint64), ("loss_scale", ctypes.c_float), ("b_offset", c_int32),
-        ("trace", c_void_p),
+        ("trace", c_void_p), ("resp_len", c_void_p),
     ]
 
 

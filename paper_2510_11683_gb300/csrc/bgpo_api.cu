@@ -171,7 +171,8 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
   if ((st = check_sample(prob, j)) != BGPO_OK) return st;
   WsLayout L;
   if ((st = check_ws(prob, ws, ws_bytes, &L)) != BGPO_OK) return st;
-  if (t_out && !aligned(t_out, 4)) return BGPO_ERR_ALIGNMENT;
+  if ((t_out && !aligned(t_out, 4)) || (prob->resp_len && !aligned(prob->resp_len, 4)))
+    return BGPO_ERR_ALIGNMENT;
   int sms = 0;
   if ((st = device_sms(&sms)) != BGPO_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -186,6 +187,7 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
   a.t_mode = prob->t_mode;
   a.t_out = t_out;
   a.mask_out = mask_out;
+  a.resp_len = prob->resp_len;
   TraceScope ts(prob->trace, KID_MASK_COMPACT, s);
   return from_cuda(launch_mask_compact(a, w, s));
 }

@@ -34,6 +34,7 @@ struct MaskArgs {
   int32_t B, R, j, n_t, t_mode;
   float* t_out;       // may be null
   uint8_t* mask_out;  // may be null
+  const int32_t* resp_len;  // may be null: [B] real response lengths
 };
 
 cudaError_t launch_mask_compact(const MaskArgs& a, const WsPtrs& w, cudaStream_t s);

@@ -173,6 +173,7 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   a.t_mode = prob->t_mode;
   a.t_out = t_out;
   a.mask_out = nullptr;
+  a.resp_len = prob->resp_len;
   CUtensorMap map_xm, map_w;
   if (!encode_map(&map_xm, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
       !encode_map(&map_w, W, g.H, g.V, g.H * 2, kBK, kBNHalf))

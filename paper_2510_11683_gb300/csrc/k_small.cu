@@ -52,6 +52,7 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
       b = (int32_t)(e / Q);
       q = (int32_t)(e % Q);
       const uint64_t bg = (uint64_t)b + (uint64_t)a.b_offset;   // global sequence index
+      const int32_t len = a.resp_len ? min(max(a.resp_len[b], 0), a.R) : a.R;
       const PhiloxOut ot = philox4x64_10(0, bg, (uint64_t)a.j, kStreamT, a.seed, 0);
       const uint64_t u = ot.w[0] >> kU24Shift;
       const uint64_t T = (a.t_mode == 1) ? ((uint64_t)a.j << 24) + u + 1 : u + 1;
@@ -60,8 +61,9 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
       for (int k = 0; k < 4; ++k) {
         const int32_t i = 4 * q + k;
         if (i < a.R) {
-          // u24 / 2^24 < T / D  <=>  u24 * (D / 2^24) < T   (exact integers)
-          const uint32_t bit = ((om.w[k] >> kU24Shift) * d_over_2_24 < T) ? 1u : 0u;
+          // u24 / 2^24 < T / D  <=>  u24 * (D / 2^24) < T   (exact integers);
+          // padding positions (i >= len) are never masked
+          const uint32_t bit = (i < len && (om.w[k] >> kU24Shift) * d_over_2_24 < T) ? 1u : 0u;
           bits |= bit << k;
           cnt += (int32_t)bit;
           if (a.mask_out) a.mask_out[(int64_t)b * a.R + i] = (uint8_t)bit;

@@ -29,12 +29,12 @@ def oracle_advantages(wl, inp):
     return O.group_advantage(to64(inp["rewards"]), wl.G)
 
 
-def oracle_run(wl, inp, loss_scale=None, b_offset=0):
+def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None):
     """Algorithm 1 inner loops in fp64: draws, l_self, l_old = l_self + eps, bound, grads."""
     X, W, Y = to64(inp["X"]), to64(inp["W"]), to64(inp["Y"])
     ls = 1.0 / wl.G if loss_scale is None else loss_scale
     A = oracle_advantages(wl, inp)
-    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode, b_offset)
+    ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode, b_offset, resp_len)
     ell_self = O.elbo_all(X, W, Y, wl.P, ts, masks)
     ell_old = ell_self + to64(inp["eps"])
     out = O.bgpo_step(X, W, Y, wl.P, A, ell_old, ts, masks, ls)
@@ -42,7 +42,7 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0):
     return out
 
 
-def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0):
+def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
@@ -51,7 +51,11 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0):
     import torch
     import paper_2510_11683_gb300 as bg
 
-    prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset)
+    lens = None
+    if resp_len is not None:
+        lens = torch.as_tensor(np.asarray(resp_len), dtype=torch.int32, device=dev)
+    prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
+                           resp_len=lens)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     B, n_t = wl.B, wl.n_t
@@ -80,7 +84,7 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0):
         bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
     torch.cuda.synchronize()
     return dict(ell=ell.T, ell_old=ell_old.T, coef=coef.T, g=g.T, t=t, masks=masks, A=A,
-                dX=dX, dW=dW, ws=ws, prob=prob, ell_self=ell_self.T)
+                dX=dX, dW=dW, ws=ws, prob=prob, ell_self=ell_self.T, lens=lens)
 
 
 def rel_ell_err(got, ref):

@@ -53,9 +53,10 @@ def test_abi_version_and_names(L, bg):
 
 
 def test_problem_struct_layout(bg):
-    assert ctypes.sizeof(bg.BgpoProblem) == 56
+    assert ctypes.sizeof(bg.BgpoProblem) == 64
     assert bg.BgpoProblem.seed.offset == 32
     assert bg.BgpoProblem.trace.offset == 48
+    assert bg.BgpoProblem.resp_len.offset == 56
 
 
 def _prob(bg, **kw):

@@ -319,3 +319,21 @@ def test_bounded_wait_times_out_and_context_survives(bg):
     torch.cuda.synchronize()
     assert bg.get_device_error(ws) == (0, 0)
     assert torch.isfinite(ell).all()
+
+
+def test_variable_length_responses(bg):
+    """Padded batches: positions at or past resp_len[b] are never masked and get
+    no gradient; everything else matches the oracle on the same draws."""
+    wl = CONFIGS["ragged"]
+    inp = make_inputs(wl, device="cuda")
+    lens = np.array([301, 0, 117])
+    g = gpu_run(wl, inp, resp_len=lens)
+    o = oracle_run(wl, {k: (v.cpu() if v is not None else None) for k, v in inp.items()},
+                   resp_len=lens)
+    assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+    assert not g["masks"][:, 1].any() and not g["masks"][:, 2, 117:].any()
+    assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= ELL_TOL
+    assert np.array_equal(to64(g["ell"])[1], np.zeros(wl.n_t))
+    assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL
+    assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL
+    assert float(g["dX"][2, 117:].abs().max()) == 0.0
