@@ -285,12 +285,14 @@ def main():
     else:
         bg.group_advantage(prob, inp["rewards"], A)
 
-    # old-policy pass (outside the timed step): l_old on the same draws (Eq. 10)
+    # old-policy pass (outside the timed step, forward only, keeps no logits):
+    # l_old on the same draws (Eq. 10)
+    prob_old = bg.problem_from(wl, b_offset=b_offset, recompute_logits=True)
     ell_old = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
     masks = torch.empty((n_t, Bsz, wl.R), dtype=torch.uint8, device=dev)
     for j in range(n_t):
-        bg.sample_mask(prob, j, ws, None, masks[j])
-        bg.elbo_fwd(prob, j, X, W, Y, ws, ell_old[j])
+        bg.sample_mask(prob_old, j, ws, None, masks[j])
+        bg.elbo_fwd(prob_old, j, X, W, Y, ws, ell_old[j])
     ell_old += inp["eps"].T.to(dev)
     masked_per_step = int(masks.sum().item())
     rows_per_sample = masks.reshape(n_t, -1).sum(dim=1).tolist()
@@ -350,9 +352,10 @@ def main():
 
     peaks = load_peaks()
     H, V = wl.H, wl.V
-    gemm_flops_per_step = 2.0 * H * V * masked_per_step   # each of the four GEMMs
-    gemm_kernels = ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
-    dom = max(gemm_kernels, key=lambda k: per_kernel.get(k, [0, 0.0])[1])
+    gemm_flops_per_step = 2.0 * H * V * masked_per_step   # each GEMM kind of the step
+    gemm_kernels = [k for k in ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
+                    if k in per_kernel]
+    dom = max(gemm_kernels, key=lambda k: per_kernel[k][1])
     dom_launches, dom_ms = per_kernel[dom]
     dom_flops_per_launch = gemm_flops_per_step * args.steps / dom_launches
     dom_avg_s = dom_ms / dom_launches / 1e3
@@ -365,20 +368,33 @@ def main():
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
                 "flops_per_launch": dom_flops_per_launch, "avg_launch_ms": dom_avg_s * 1e3}
 
+    # dL/dz from the kept logits: reads 4 V and writes 2 V bytes per masked row
+    hbm_pass = None
+    if "dz_from_logits" in per_kernel:
+        n_dz, dz_ms = per_kernel["dz_from_logits"]
+        dz_bytes = 6.0 * V * masked_per_step * args.steps / n_dz
+        dz_gbs = dz_bytes / (dz_ms / n_dz / 1e3) / 1e9
+        hbm_pass = {"kernel": "dz_from_logits", "bound": "hbm", "achieved": dz_gbs,
+                    "peak": peaks["hbm"], "unit": "GB/s", "frac": dz_gbs / peaks["hbm"],
+                    "bytes_per_launch": dz_bytes, "avg_launch_ms": dz_ms / n_dz,
+                    "peak_kind": f"HBM copy ({peaks['source']})"}
+
     value = masked_all / (ms / 1e3)
-    exec_tflops = 4 * gemm_flops_per_step / (ms / 1e3) / 1e12
+    exec_tflops = len(gemm_kernels) * gemm_flops_per_step / (ms / 1e3) / 1e12
+    useful_tflops = 3 * gemm_flops_per_step / (ms / 1e3) / 1e12   # fwd, dX, dW
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; shapes of the paper's "
         "LLaDA-8B head, response 512, n_t=16)", "config": config_of(wl),
-        "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clock_info,
+        "roofline": roofline, "roofline_hbm_pass": hbm_pass, "gpu_launches": gpu_launches,
+        "clocks": clock_info,
         "mc_samples_per_s": Bsz * n_t * world / (ms / 1e3),
         "masked_rows_per_step": masked_per_step, "masked_rows_per_sample": rows_per_sample,
         "step_tensor_tflops_executed": exec_tflops,
         "step_frac_of_bf16_peak_executed": exec_tflops / peaks["bf16"],
-        "step_frac_of_bf16_peak_useful": 0.75 * exec_tflops / peaks["bf16"],
+        "step_frac_of_bf16_peak_useful": useful_tflops / peaks["bf16"],
         "per_kernel_ms_per_step": {k: v[1] / args.steps for k, v in per_kernel.items()},
         "peak_mem_bytes": torch.cuda.max_memory_allocated(dev),
         "workspace_bytes": ws.numel(),
@@ -570,7 +586,9 @@ def nt_sweep(bg, dev):
     """Time and peak memory of one step vs n_t (8 x (256 + 512), LLaDA-8B head) for
     BGPO and for the ELBO-based objective it bounds (VRPO, Eq. 7), whose weights
     need every sample's l first: "vrpo_retain" keeps one workspace per sample
-    (memory grows with n_t), "vrpo_recompute" runs each sample's forward twice."""
+    (memory grows with n_t), "vrpo_recompute" runs each sample's forward twice.
+    Every backward reads logits its forward kept (the default mode); the first,
+    forward-only pass of "vrpo_recompute" keeps none."""
     import torch
     from synth import CONFIGS, SWEEP_NT, make_inputs
     base = CONFIGS["llada8b_sweep"]
@@ -581,6 +599,7 @@ def nt_sweep(bg, dev):
     for n_t in SWEEP_NT:
         wl = base.with_(n_t=n_t)
         prob = bg.problem_from(wl)
+        prob_lean = bg.problem_from(wl, recompute_logits=True)
         A = torch.empty(wl.B, dtype=torch.float32, device=dev)
         bg.group_advantage(prob, rewards, A)
         rows = 0
@@ -613,10 +632,11 @@ def nt_sweep(bg, dev):
                         bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
                         bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
                     return
+                p1 = prob if method == "vrpo_retain" else prob_lean
                 for j in range(n_t):
                     ws = wss[j % n_ws]
-                    bg.sample_mask(prob, j, ws)
-                    bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
+                    bg.sample_mask(p1, j, ws)
+                    bg.elbo_fwd(p1, j, X, W, Y, ws, ell[j])
                 bg.vrpo_coeffs(prob, ell, ell, A, cv, None, wss[0])
                 for j in range(n_t):
                     ws = wss[j % n_ws]

@@ -8,7 +8,8 @@
  *   bgpo_sample_mask          t_{b,j} and the response mask (Sec. 2.1; Eq. 3, 5;
  *                             Algorithm 1, sampling of t and y_t)
  *   bgpo_elbo_fwd             l_{b,j} = (1/t) sum_masked log p(y^i | y_t, x) through
- *                             the LM head (Eq. 4), full logits never stored
+ *                             the LM head (Eq. 4); the masked rows' logits are
+ *                             kept in the workspace for the backward
  *   bgpo_bound_coeffs         d_j (Eq. 10), g_j (Eq. 13) and dL_j/dl_j with
  *                             L_j = -loss_scale * g_j (Algorithm 1; Eq. 19)
  *   bgpo_elbo_bwd_accumulate  dX += dL_j/dX, dW += dL_j/dW (Algorithm 1, gradient
@@ -33,7 +34,8 @@
  *  - Alignment: X, W, dX, dW and the workspace must be 16-byte aligned
  *    (workspace: 256-byte). H must be a multiple of 64.
  *  - The workspace carries sample j's draws (t, mask), its compacted masked
- *    rows and forward statistics from one call to the next, so the calls for
+ *    rows, forward statistics and (unless BGPO_FLAG_RECOMPUTE_LOGITS is set)
+ *    the masked rows' logits from one call to the next, so the calls for
  *    one sample must be issued in the order
  *        bgpo_sample_mask -> bgpo_elbo_fwd -> [bgpo_bound_coeffs] ->
  *        bgpo_elbo_bwd_accumulate
@@ -57,7 +59,7 @@
 extern "C" {
 #endif
 
-#define BGPO_ABI_VERSION 1
+#define BGPO_ABI_VERSION 2
 
 typedef enum bgpo_status {
   BGPO_OK = 0,
@@ -79,6 +81,19 @@ typedef struct bgpo_trace bgpo_trace;
 #define BGPO_T_STRATIFIED 1  /* t_{b,j} in (j/n_t, (j+1)/n_t]; not in the paper */
 
 /*
+ * flags bits
+ *   BGPO_FLAG_RECOMPUTE_LOGITS  bgpo_elbo_fwd keeps no logits; the backward of
+ *       that sample recomputes them with a fourth tensor-core GEMM. Without the
+ *       flag (the default) the forward writes the fp32 logits z = Xm W^T of the
+ *       masked rows into the workspace and the backward forms dL/dz from them
+ *       in one HBM-bound pass: same results bit for bit, about a quarter less
+ *       tensor-core work per sample, 4 * roundup(B R, 256) * roundup(V, 64)
+ *       more workspace bytes. Set it for forward-only passes (the old policy's
+ *       l_old) or to save memory.
+ */
+#define BGPO_FLAG_RECOMPUTE_LOGITS 1u
+
+/*
  * Problem description (host struct, read by every call; never stored).
  *   B      responses in the batch (>= 1)
  *   P      prompt length: X rows [b, 0, P) are the prompt, never masked (Sec. 2.1)
@@ -98,6 +113,8 @@ typedef struct bgpo_trace bgpo_trace;
  *          response b holds resp_len[b] tokens (0 <= resp_len[b] <= R); positions
  *          i >= resp_len[b] are padding and never masked (the draws of the other
  *          positions are unchanged; values outside [0, R] are clamped)
+ *   flags  BGPO_FLAG_* bits (0 = defaults); other bits are rejected
+ *   reserved  must be 0
  * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
  * bgpo_workspace_bytes).
  */
@@ -115,6 +132,8 @@ typedef struct bgpo_problem {
   int32_t b_offset;
   bgpo_trace* trace;
   const int32_t* resp_len;
+  uint32_t flags;
+  int32_t reserved;
 } bgpo_problem;
 
 /* ABI version of the loaded library (BGPO_ABI_VERSION). */
@@ -126,14 +145,16 @@ const char* bgpo_status_string(bgpo_status status);
 /*
  * Host-only validation of a problem description (no CUDA call).
  * Returns BGPO_OK, BGPO_ERR_INVALID_ARG (NULL, bad t_mode, negative b_offset,
- * non-finite loss_scale) or BGPO_ERR_SHAPE.
+ * non-finite loss_scale, unknown flags, non-zero reserved) or BGPO_ERR_SHAPE.
  */
 bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
 
 /*
  * Bytes of device workspace the calls below need for `prob`. Depends on B, R,
- * H and V only -- never on n_t (Linearity, Sec. 3: one sample's state at a
- * time). Returns 0 for an invalid problem.
+ * H, V and BGPO_FLAG_RECOMPUTE_LOGITS only -- never on n_t (Linearity, Sec. 3:
+ * one sample's state at a time). The layout without the logits is a prefix of
+ * the layout with them, so a workspace sized without the flag also serves
+ * calls made with it. Returns 0 for an invalid problem.
  */
 size_t bgpo_workspace_bytes(const bgpo_problem* prob);
 
@@ -162,7 +183,9 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
  * (no length normalisation; an empty mask gives 0). The masked rows of X are
  * gathered, multiplied by W on the tensor cores (bf16 in, fp32 accumulate)
  * and reduced by an online log-sum-exp per row; the per-row log-sum-exp and
- * log-probabilities stay in the workspace for the backward pass. The result is
+ * log-probabilities stay in the workspace for the backward pass, and so do the
+ * fp32 logits of the masked rows unless BGPO_FLAG_RECOMPUTE_LOGITS is set
+ * (full logits are never written to caller memory). The result is
  * deterministic (fixed reduction order), so recomputing l with unchanged inputs
  * gives bit-identical values (on-policy d_j = 0 exactly, Sec. 3.2).
  *   X      device bf16 [B, P+R, H];  W device bf16 [V, H];  Y device int32 [B, R]
@@ -209,13 +232,19 @@ bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const f
  * Backward pass of L_j = sum_b coef_b * l_{b,j}, accumulated (Algorithm 1,
  * gradient accumulation; Eq. 15-17 give the per-sample gradient weights):
  *   w_r   = coef_b / t_{b,j}                       for masked row r = (b, i)
- *   dz_r  = w_r (onehot(Y[b,i]) - softmax(W x_r))  (logits recomputed; bf16)
+ *   dz_r  = w_r (onehot(Y[b,i]) - softmax(W x_r))  (bf16; the softmax comes
+ *           from the logits bgpo_elbo_fwd kept, or with BGPO_FLAG_RECOMPUTE_LOGITS
+ *           from logits recomputed on the tensor cores; the two give identical
+ *           bits)
  *   dX[b, i, :] += W^T dz_r        dW += sum_r dz_r x_r^T
  * coef is an input (normally bgpo_bound_coeffs' output for the same j).
  *   dX device float [B, R, H], dW device float [V, H]: accumulated in place.
  * Deterministic: no atomics, fixed summation order.
  * Requires bgpo_sample_mask(j) and bgpo_elbo_fwd(j) before it on the same
- * workspace, with the same X, W and Y.
+ * workspace, with the same X, W and Y. Without BGPO_FLAG_RECOMPUTE_LOGITS the
+ * last bgpo_elbo_fwd of sample j must have kept its logits (been called without
+ * the flag); otherwise the device error word is set to BGPO_ERR_INVALID_ARG and
+ * dX and dW are left unchanged.
  */
 bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
                                      const void* W, const int32_t* Y, const float* coef, void* ws,
@@ -240,6 +269,7 @@ bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards,
  * need.
  *   X, W, Y   as for bgpo_elbo_fwd;  t_out device float [B] or NULL;
  *   ell_out   device float [B]: l_{b,j} (Eq. 4), same values as bgpo_elbo_fwd.
+ * It keeps no logits (prob->flags is validated, then ignored).
  * Limit: the forward scratch of `prob` must fit the 32 MiB array, about
  * roundup(B*R, 128) * (2 H + 8 ceil(V / 256) + 20) bytes; larger problems
  * return BGPO_ERR_WORKSPACE_TOO_SMALL before anything is launched.

@@ -55,6 +55,7 @@ bgpo_status check_problem(const bgpo_problem* p) {
   if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
   if (p->b_offset < 0) return BGPO_ERR_INVALID_ARG;
   if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
+  if ((p->flags & ~BGPO_FLAG_RECOMPUTE_LOGITS) != 0u || p->reserved != 0) return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
   if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
@@ -66,6 +67,8 @@ bgpo_status check_problem(const bgpo_problem* p) {
 
 Geometry geometry_of(const bgpo_problem* p) { return make_geometry(p->B, p->P, p->R, p->H, p->V); }
 
+bool keeps_logits(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_RECOMPUTE_LOGITS) == 0u; }
+
 bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
   return (j >= 0 && j < p->n_t) ? BGPO_OK : BGPO_ERR_INVALID_ARG;
 }
@@ -73,7 +76,7 @@ bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
 bgpo_status check_ws(const bgpo_problem* p, const void* ws, size_t ws_bytes, WsLayout* L) {
   if (!ws) return BGPO_ERR_INVALID_ARG;
   if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
-  *L = make_ws_layout(geometry_of(p));
+  *L = make_ws_layout(geometry_of(p), keeps_logits(p));
   if (ws_bytes < L->total) return BGPO_ERR_WORKSPACE_TOO_SMALL;
   return BGPO_OK;
 }
@@ -161,7 +164,7 @@ bgpo_status bgpo_validate_problem(const bgpo_problem* prob) { return check_probl
 
 size_t bgpo_workspace_bytes(const bgpo_problem* prob) {
   if (check_problem(prob) != BGPO_OK) return 0;
-  return make_ws_layout(geometry_of(prob)).total;
+  return make_ws_layout(geometry_of(prob), keeps_logits(prob)).total;
 }
 
 bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size_t ws_bytes,
@@ -209,9 +212,13 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
   const Geometry g = geometry_of(prob);
   const WsPtrs w = ws_pointers(ws, L);
 
-  CUtensorMap map_xm, map_w;
+  const bool keep = w.zc != nullptr;
+  CUtensorMap map_xm, map_w, map_zc;
   if (!map_2d(&map_xm, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
-      !map_2d(&map_w, W, g.H, g.V, g.H * 2, kBK, kBNHalf))
+      !map_2d(&map_w, W, g.H, g.V, g.H * 2, kBK, kBNHalf) ||
+      // logits leave the epilogue as 32-row x 32-column fp32 sub-tiles
+      (keep && !map_2d(&map_zc, w.zc, g.v_pad, g.m_pad, g.v_pad * 4, 32, 32,
+                       CU_TENSOR_MAP_DATA_TYPE_FLOAT32)))
     return BGPO_ERR_CUDA;
   GemmArgs ga;
   ga.g = g;
@@ -225,11 +232,12 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
   }
   {
     TraceScope ts(prob->trace, KID_LMHEAD_FWD, s);
-    if (launch_gemm(GEMM_FWD, map_xm, map_w, map_xm, ga, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_gemm(GEMM_FWD, map_xm, map_w, keep ? map_zc : map_xm, ga, w, s) != cudaSuccess)
+      return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_LSE_COMBINE, s);
-    if (launch_lse_combine(g, j, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_lse_combine(g, j, keep, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_SEQ_REDUCE, s);
@@ -297,6 +305,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   const Geometry g = geometry_of(prob);
   const WsPtrs w = ws_pointers(ws, L);
 
+  const bool keep = w.zc != nullptr;
   CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xm_mn;
   CUtensorMap map_dz_st, map_dxp_st, map_dw_red;
   const uint64_t dxp_rows = (uint64_t)dxp_row_block_cap(g) * kPairM;
@@ -317,7 +326,10 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   ga.j = j;
   ga.coef = coef;
   ga.dW = dW;
-  {
+  if (keep) {
+    TraceScope ts(prob->trace, KID_DZ_FROM_LOGITS, s);
+    if (launch_dz_from_logits(g, j, coef, sms, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  } else {
     TraceScope ts(prob->trace, KID_LMHEAD_DZ, s);
     if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, map_dz_st, ga, w, s) != cudaSuccess)
       return BGPO_ERR_CUDA;
@@ -442,7 +454,7 @@ const char* bgpo_kernel_name(int32_t id) {
   static const char* names[KID_COUNT] = {
       "mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
       "bound_coeffs", "lmhead_dz",   "dx_gemm",        "dx_reduce",   "dw_gemm",
-      "group_advantage", "selftest_wait", "vrpo_coeffs"};
+      "group_advantage", "selftest_wait", "vrpo_coeffs", "dz_from_logits"};
   return (id >= 0 && id < KID_COUNT) ? names[id] : "?";
 }
 

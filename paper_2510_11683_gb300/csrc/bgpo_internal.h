@@ -24,6 +24,7 @@ struct WsPtrs {
   void* xm;   // bf16
   void* dz;   // bf16
   float* dxp;
+  float* zc;  // fp32 logits kept by the forward; null when the layout has none
 };
 
 WsPtrs ws_pointers(void* ws, const WsLayout& L);
@@ -40,7 +41,12 @@ struct MaskArgs {
 cudaError_t launch_mask_compact(const MaskArgs& a, const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_gather(const Geometry& g, int32_t j, const void* X, const int32_t* Y,
                           const WsPtrs& w, cudaStream_t s);
-cudaError_t launch_lse_combine(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s);
+// `kept_logits`: the forward GEMM just wrote this sample's logits to w.zc.
+cudaError_t launch_lse_combine(const Geometry& g, int32_t j, bool kept_logits, const WsPtrs& w,
+                               cudaStream_t s);
+// dz from the logits the forward kept (same arithmetic as the GEMM_DZ epilogue).
+cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, const float* coef, int num_sms,
+                                  const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* ell_out,
                               cudaStream_t s);
 cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
@@ -71,8 +77,9 @@ struct GemmArgs {
 // grid is resident.
 int gemm_num_pairs(int num_sms);
 
-// map_a / map_b: the operand tiles; map_c: the epilogue's destination (dZ for
-// GEMM_DZ, the split-K partials for GEMM_DX, dW for GEMM_DW; unused by GEMM_FWD).
+// map_a / map_b: the operand tiles; map_c: the epilogue's destination (the
+// fp32 logit region for GEMM_FWD when w.zc is set, dZ for GEMM_DZ, the split-K
+// partials for GEMM_DX, dW for GEMM_DW).
 cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorMap& map_b,
                         const CUtensorMap& map_c, const GemmArgs& a, const WsPtrs& w,
                         cudaStream_t s);

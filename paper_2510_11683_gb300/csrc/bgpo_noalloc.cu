@@ -91,6 +91,8 @@ FwdLayout forward_layout(const Geometry& g) {
   L.dz = 0;
   L.dxp = 0;
   L.dxp_elems = 0;
+  L.zc = 0;        // keeps no logits
+  L.zc_bytes = 0;
   L.total = o;
   f.total = o;
   return f;
@@ -187,7 +189,7 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   if (launch_mask_compact(a, w, s) != cudaSuccess ||
       launch_gather(g, j, X, Y, w, s) != cudaSuccess ||
       launch_gemm(GEMM_FWD, map_xm, map_w, map_xm, ga, w, s) != cudaSuccess ||
-      launch_lse_combine(g, j, w, s) != cudaSuccess ||
+      launch_lse_combine(g, j, false, w, s) != cudaSuccess ||
       launch_seq_reduce(g, j, w, ell_out, s) != cudaSuccess)
     return BGPO_ERR_CUDA;
   return BGPO_OK;

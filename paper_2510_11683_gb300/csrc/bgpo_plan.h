@@ -49,7 +49,8 @@ enum KernelId : int32_t {
   KID_GROUP_ADV = 10,
   KID_SELFTEST_WAIT = 11,
   KID_VRPO_COEFFS = 12,
-  KID_COUNT = 13
+  KID_DZ_FROM_LOGITS = 13,
+  KID_COUNT = 14
 };
 
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -105,7 +106,7 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
 // Device workspace layout. Every region starts on a 1024-byte boundary (TMA
 // tiles with 128-byte swizzle want 1024-byte aligned bases).
 struct WsLayout {
-  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M
+  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M, [4] logits kept
   size_t t;          // float[B]    t_{b,j}
   size_t tnum;       // uint32[2B]  T numerator (t = T / D), (low, high) words
   size_t seg_off;    // int32[B+1]  first compacted row of each sequence
@@ -119,6 +120,8 @@ struct WsLayout {
   size_t dz;         // bf16[m_pad * v_pad] dL/dz of the current sample
   size_t dxp;        // float[dxp_elems] split-K partials of dX
   size_t dxp_elems;
+  size_t zc;         // float[m_pad * v_pad] logits kept by the forward (last region)
+  size_t zc_bytes;   // 0 when the forward keeps no logits
   size_t total;
 };
 
@@ -131,7 +134,9 @@ BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
   return mb_max > kMaxSplits ? mb_max : kMaxSplits;
 }
 
-BGPO_HD WsLayout make_ws_layout(const Geometry& g) {
+// `keep_logits` appends the fp32 logit region; every other region has the same
+// offset either way.
+BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
   WsLayout L;
   size_t o = 0;
   L.err = o;       o = align_ws(o + 64);
@@ -148,11 +153,16 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g) {
   L.dz = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.v_pad);
   L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;
   L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
+  L.zc_bytes = keep_logits ? 4 * (size_t)g.m_pad * (size_t)g.v_pad : 0;
+  L.zc = keep_logits ? o : 0;
+  o = align_ws(o + L.zc_bytes);
   L.total = o;
   return L;
 }
 
-// Indices into the int32 error word.
-enum ErrField : int { ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3 };
+// Indices into the int32 error word. ERR_LOGITS is 1 while the logit region
+// holds the current sample's logits (set by the forward that wrote them,
+// cleared by the masking of a new sample and by a forward that keeps none).
+enum ErrField : int { ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4 };
 
 }  // namespace bgpo

@@ -18,10 +18,12 @@
 //
 // Kinds (Xm = gathered masked hidden states [M, H], W = LM head [V, H]):
 //   GEMM_FWD  z = Xm W^T; epilogue: online max / sum-exp per (row, vocab tile)
-//             and the target logit (Eq. 4: log softmax gathered at y^i); full
-//             logits are never written.
-//   GEMM_DZ   z = Xm W^T recomputed; epilogue: dz = w_r (onehot - e^{z - lse})
-//             stored as bf16 (gradient of Eq. 4 weighted by Eq. 13's dL/dl).
+//             and the target logit (Eq. 4: log softmax gathered at y^i); when
+//             the workspace has a logit region the fp32 tile also leaves
+//             through TMA stores, for the backward.
+//   GEMM_DZ   z = Xm W^T recomputed (when the forward kept no logits);
+//             epilogue: dz = w_r (onehot - e^{z - lse}) stored as bf16
+//             (gradient of Eq. 4 weighted by Eq. 13's dL/dl).
 //   GEMM_DX   dXm = dZ W (K = vocabulary, split-K partials in fp32).
 //   GEMM_DW   dW += dZ^T Xm (K = masked rows), fp32 TMA reduce-add.
 //
@@ -122,13 +124,13 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
   return t;
 }
 
-// Shared-memory plan of one kind: the forward GEMM writes no tiles from its
-// epilogue and needs no staging space (a 7th stage in that space measured no
-// faster than 6).
+// Shared-memory plan of one kind: 6 pipeline stages and the epilogue's
+// staging buffers (the forward GEMM stages its fp32 logits there when it keeps
+// them).
 template <int KIND>
 struct SmemPlan {
   static constexpr int stages = kStages;
-  static constexpr uint32_t epi_bytes = (KIND == GEMM_FWD) ? 0u : kEpiBytes;
+  static constexpr uint32_t epi_bytes = kEpiBytes;
   static constexpr uint32_t bytes = stages * kStageBytes + epi_bytes + 1024 + 1024;
   static_assert(bytes <= 232448, "shared memory per CTA");
 };
@@ -199,47 +201,6 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 // ---- epilogues: one thread per accumulator row; row0 = first row of the warp --------
 
-// GEMM_FWD: per (row, vocab tile) the pair (max z, sum e^{z - max}) and, in the
-// tile holding y_r, the target logit z_{r, y_r}.
-__device__ __forceinline__ void epi_fwd(const GemmParams& p, int32_t M, const Unit& t,
-                                        int64_t row0, int lane, uint32_t tb) {
-  const int64_t r = row0 + lane;
-  const bool valid = r < M;
-  const int32_t y = valid ? p.w.tgt[r] : -1;
-  const int32_t v0 = t.n_blk * kBN;
-  const int32_t V = (int32_t)p.g.V;
-  float m = -INFINITY, s = 0.f, tl = 0.f;
-  bool hit = false;
-#pragma unroll 1
-  for (int c = 0; c < kBN / 32; ++c) {
-    const int32_t col0 = v0 + c * 32;
-    if (col0 >= V) break;  // warp-uniform
-    uint32_t raw[32];
-    tmem_ld_32x32b_x32(tb + c * 32, raw);
-    tmem_ld_wait();
-    const int nvalid = min(32, V - col0);
-    float cm = -INFINITY;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const float z = bits_f(raw[k]);
-      if (k < nvalid) cm = fmaxf(cm, z);
-      if (col0 + k == y) { tl = z; hit = true; }
-    }
-    const float mn = fmaxf(m, cm);
-    const float mnl = mn * kLog2e;
-    float acc = 0.f;
-#pragma unroll
-    for (int k = 0; k < 32; ++k)
-      if (k < nvalid) acc += exp2f(fmaf(bits_f(raw[k]), kLog2e, -mnl));
-    s = s * exp2f((m - mn) * kLog2e) + acc;
-    m = mn;
-  }
-  if (valid) {
-    p.w.part[r * p.g.n_vt + t.n_blk] = make_float2(m, s);
-    if (hit) p.w.tgt_logit[r] = tl;
-  }
-}
-
 // Epilogue staging of one warp: two 32-row x 128-byte buffers in the 128-byte
 // swizzled layout the TMA tensor maps use (16-byte chunk q of row r stored at
 // chunk q ^ (r & 7)), so that 32 lanes writing one row each hit 8 bank groups.
@@ -276,6 +237,58 @@ __device__ __forceinline__ void stage_row(uint32_t sbuf, int lane, const uint4 (
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(chunk[q].x),
                  "r"(chunk[q].y), "r"(chunk[q].z), "r"(chunk[q].w)
                  : "memory");
+  }
+}
+
+// GEMM_FWD: per (row, vocab tile) the pair (max z, sum e^{z - max}) and, in the
+// tile holding y_r, the target logit z_{r, y_r}; with a logit region, the
+// fp32 logits too (32-column sub-tiles through TMA stores into [m_pad, v_pad]).
+__device__ __forceinline__ void epi_fwd(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
+                                        const Unit& t, int64_t row0, int lane, uint32_t tb,
+                                        EpiStage& st) {
+  const int64_t r = row0 + lane;
+  const bool valid = r < M;
+  const int32_t y = valid ? p.w.tgt[r] : -1;
+  const int32_t v0 = t.n_blk * kBN;
+  const int32_t V = (int32_t)p.g.V;
+  float m = -INFINITY, s = 0.f, tl = 0.f;
+  bool hit = false;
+#pragma unroll 1
+  for (int c = 0; c < kBN / 32; ++c) {
+    const int32_t col0 = v0 + c * 32;
+    if (col0 >= V) break;  // warp-uniform
+    uint32_t raw[32];
+    tmem_ld_32x32b_x32(tb + c * 32, raw);
+    tmem_ld_wait();
+    const int nvalid = min(32, V - col0);
+    float cm = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float z = bits_f(raw[k]);
+      if (k < nvalid) cm = fmaxf(cm, z);
+      if (col0 + k == y) { tl = z; hit = true; }
+    }
+    const float mn = fmaxf(m, cm);
+    const float mnl = mn * kLog2e;
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 32; ++k)
+      if (k < nvalid) acc += exp2f(fmaf(bits_f(raw[k]), kLog2e, -mnl));
+    s = s * exp2f((m - mn) * kLog2e) + acc;
+    m = mn;
+    if (p.w.zc != nullptr) {  // kernel-uniform; col0 < V <= v_pad, both multiples of 32
+      uint4 chunk[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
+      const uint32_t sbuf = st.acquire(lane);
+      stage_row(sbuf, lane, chunk);
+      st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, col0, (int32_t)row0); });
+    }
+  }
+  if (valid) {
+    p.w.part[r * p.g.n_vt + t.n_blk] = make_float2(m, s);
+    if (hit) p.w.tgt_logit[r] = tl;
   }
 }
 
@@ -402,7 +415,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* s_a = smem;
   uint8_t* s_b = smem + kSt * kTileABytes;
-  uint8_t* s_epi = s_b + kSt * kTileBBytes;   // 4 warps x 2 staging buffers (not GEMM_FWD)
+  uint8_t* s_epi = s_b + kSt * kTileBBytes;   // 4 warps x 2 staging buffers
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_epi + SmemPlan<KIND>::epi_bytes);
   uint64_t* full = bars;                      // [kSt] TMA (both CTAs) -> MMA; even CTA's
   uint64_t* empty = bars + kSt;           // [kSt] MMA -> TMA of each CTA
@@ -447,7 +460,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&map_a);
     tma_prefetch_map(&map_b);
-    if (KIND != GEMM_FWD) tma_prefetch_map(&map_c);
+    tma_prefetch_map(&map_c);
   }
   if (warp == 1) {
     tmem_alloc_pair(smem_addr(tmem_slot), kTmemCols);
@@ -558,7 +571,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN);
       const int64_t row0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM + quarter * 32;
-      if (KIND == GEMM_FWD) epi_fwd(p, M, t, row0, lane, tb);
+      if (KIND == GEMM_FWD) epi_fwd(p, &map_c, M, t, row0, lane, tb, st);
       else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, lane, tb, st);
       else if (KIND == GEMM_DX) epi_dx(p, &map_c, wk, t, row0, lane, tb, st);
       else epi_dw(p, &map_c, t, row0, lane, tb, st);

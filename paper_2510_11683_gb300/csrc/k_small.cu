@@ -1,7 +1,8 @@
 // Non-GEMM kernels of the BGPO LM-head ELBO path: the forward masking process
 // with row compaction, the gather of masked hidden states, the log-sum-exp
 // combine, the per-sequence ELBO reduction (Eq. 4), the bound coefficients
-// (Eq. 10, 13), the split-K reduction of dX and the group advantages (Eq. 18).
+// (Eq. 10, 13), dL/dz from the logits the forward kept, the split-K reduction
+// of dX and the group advantages (Eq. 18).
 #include <math.h>
 
 #include "bgpo_device.cuh"
@@ -14,6 +15,7 @@ namespace {
 
 constexpr int32_t kStatusInvalidArg = 1;   // BGPO_ERR_INVALID_ARG
 constexpr int32_t kStatusNonfinite = 5;    // BGPO_ERR_NONFINITE
+constexpr float kLog2e = 1.4426950408889634f;
 
 // Masked rows of the sample the workspace holds, or 0 (and an error) when the
 // workspace holds another sample than `j`.
@@ -114,6 +116,7 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
     w.seg_off[a.B] = M;
     w.err[ERR_M] = M;
     w.err[ERR_SAMPLE] = a.j;
+    w.err[ERR_LOGITS] = 0;  // no forward of this sample has kept its logits yet
   }
 }
 
@@ -156,8 +159,11 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
 // log-sum-exp of each masked row from the per-vocab-tile partials, then
 // log p(y_r) = z_{r, y_r} - lse_r. One warp per row, fixed merge order.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, WsPtrs w) {
+__global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, bool kept_logits,
+                                                     WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_LSE_COMBINE);
+  if (blockIdx.x == 0 && threadIdx.x == 0)
+    w.err[ERR_LOGITS] = (kept_logits && w.err[ERR_SAMPLE] == j) ? 1 : 0;
   const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= M) return;
@@ -177,6 +183,88 @@ __global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, WsPt
     const float lse = m + logf(s);
     w.lse[r] = lse;
     w.logp[r] = w.tgt_logit[r] - lse;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// dL/dz of the masked rows from the logits the forward kept:
+//   dz_{r,v} = w_r (1[v = y_r] - e^{z_{r,v} - lse_r}),  w_r = coef_b / t_b
+// (gradient of Eq. 4 weighted by dL/dl), bf16, zero for rows in
+// [M, round_up(M, 256)) and columns in [V, v_pad): the arithmetic of the
+// GEMM_DZ epilogue on the same fp32 logits, so both give identical bits.
+// HBM-bound: each row streams 4 v_pad bytes in and 2 v_pad bytes out. Work
+// items are (row, 8192-column chunk); each thread has kDzVec independent
+// 32-byte loads in flight before it computes.
+// When the workspace holds no logits of sample j the kernel records
+// BGPO_ERR_INVALID_ARG and invalidates the sample tag, so that the dX / dW
+// kernels after it do no work.
+// ---------------------------------------------------------------------------
+constexpr int kDzThreads = 256;
+constexpr int kDzVec = 4;                           // 8-column vectors per thread per item
+constexpr int kDzItemVecs = kDzThreads * kDzVec;    // 1024 vectors = 8192 columns
+
+__global__ void __launch_bounds__(kDzThreads, 4)
+    k_dz_from_logits(Geometry g, int32_t j, const float* __restrict__ coef, WsPtrs w) {
+  const int32_t M = rows_of_sample(w.err, j, KID_DZ_FROM_LOGITS);
+  if (w.err[ERR_LOGITS] != 1) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      set_device_error(w.err, kStatusInvalidArg, KID_DZ_FROM_LOGITS * 16 + 2);
+      w.err[ERR_SAMPLE] = -1;
+    }
+    return;
+  }
+  const int64_t nvec = g.v_pad / 8;
+  const int64_t per_row = ceil_div(nvec, kDzItemVecs);
+  const int64_t items = round_up(M, kPairM) * per_row;
+  const float4* __restrict__ zc = reinterpret_cast<const float4*>(w.zc);
+  uint4* __restrict__ dz = reinterpret_cast<uint4*>(w.dz);
+  const int32_t V = (int32_t)g.V;
+  for (int64_t q = blockIdx.x; q < items; q += gridDim.x) {
+    const int64_t r = q / per_row;
+    const int64_t v0 = (q % per_row) * kDzItemVecs + threadIdx.x;
+    const bool valid = r < M;
+    float wr = 0.f, lse_l2 = 0.f;
+    int32_t y = -1;
+    if (valid) {
+      const int32_t b = w.rows[r] / (int32_t)g.R;
+      wr = coef[b] / w.t[b];
+      lse_l2 = w.lse[r] * kLog2e;
+      y = w.tgt[r];
+    }
+    float4 z[kDzVec][2];
+#pragma unroll
+    for (int k = 0; k < kDzVec; ++k) {
+      const int64_t v = v0 + k * kDzThreads;
+      if (valid && v < nvec) {
+        const float4* src = zc + (r * nvec + v) * 2;
+        z[k][0] = __ldcs(src);
+        z[k][1] = __ldcs(src + 1);
+      } else {
+        z[k][0] = z[k][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kDzVec; ++k) {
+      const int64_t v = v0 + k * kDzThreads;
+      if (v >= nvec) continue;
+      const float zz[8] = {z[k][0].x, z[k][0].y, z[k][0].z, z[k][0].w,
+                           z[k][1].x, z[k][1].y, z[k][1].z, z[k][1].w};
+      uint32_t packed[4];
+#pragma unroll
+      for (int e = 0; e < 8; e += 2) {
+        float d[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int32_t col = (int32_t)(v * 8) + e + h;
+          const float pr = exp2f(fmaf(zz[e + h], kLog2e, -lse_l2));
+          const float val = wr * ((col == y ? 1.f : 0.f) - pr);
+          d[h] = (valid && col < V) ? val : 0.f;
+        }
+        const __nv_bfloat162 hv = __floats2bfloat162_rn(d[0], d[1]);
+        packed[e / 2] = *reinterpret_cast<const uint32_t*>(&hv);
+      }
+      dz[r * nvec + v] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    }
   }
 }
 
@@ -326,6 +414,7 @@ WsPtrs ws_pointers(void* ws, const WsLayout& L) {
   p.xm = base + L.xm;
   p.dz = base + L.dz;
   p.dxp = reinterpret_cast<float*>(base + L.dxp);
+  p.zc = L.zc_bytes ? reinterpret_cast<float*>(base + L.zc) : nullptr;
   return p;
 }
 
@@ -341,9 +430,19 @@ cudaError_t launch_gather(const Geometry& g, int32_t j, const void* X, const int
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse_combine(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s) {
+cudaError_t launch_lse_combine(const Geometry& g, int32_t j, bool kept_logits, const WsPtrs& w,
+                               cudaStream_t s) {
   const unsigned grid = (unsigned)ceil_div(g.m_cap, 8);
-  k_lse_combine<<<grid, 256, 0, s>>>(g, j, w);
+  k_lse_combine<<<grid, 256, 0, s>>>(g, j, kept_logits, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, const float* coef, int num_sms,
+                                  const WsPtrs& w, cudaStream_t s) {
+  // 4 resident CTAs per SM; never more CTAs than the largest sample has items
+  const int64_t most = g.m_pad * ceil_div(g.v_pad / 8, kDzItemVecs);
+  const int64_t grid = most < 4 * (int64_t)num_sms ? most : 4 * (int64_t)num_sms;
+  k_dz_from_logits<<<(unsigned)grid, kDzThreads, 0, s>>>(g, j, coef, w);
   return cudaGetLastError();
 }
 

@@ -42,8 +42,13 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None):
     return out
 
 
-def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None):
+def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None,
+            recompute_logits=False):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
+
+    The old-policy pass is forward-only and always runs with
+    BGPO_FLAG_RECOMPUTE_LOGITS (it keeps no logits, on the same workspace);
+    `recompute_logits` selects the mode of the inner loop.
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
     masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
@@ -55,7 +60,9 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     if resp_len is not None:
         lens = torch.as_tensor(np.asarray(resp_len), dtype=torch.int32, device=dev)
     prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                           resp_len=lens)
+                           resp_len=lens, recompute_logits=recompute_logits)
+    prob_old = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
+                               resp_len=lens, recompute_logits=True)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     B, n_t = wl.B, wl.n_t
@@ -69,8 +76,8 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     masks = torch.empty((n_t, B, wl.R), dtype=torch.uint8, device=dev)
     ell_self = torch.empty((n_t, B), dtype=torch.float32, device=dev)
     for j in range(n_t):          # old-policy pass (same draws, Eq. 10)
-        bg.sample_mask(prob, j, ws, t[j], masks[j])
-        bg.elbo_fwd(prob, j, X, W, Y, ws, ell_self[j])
+        bg.sample_mask(prob_old, j, ws, t[j], masks[j])
+        bg.elbo_fwd(prob_old, j, X, W, Y, ws, ell_self[j])
     ell_old = (ell_self + inp["eps"].T.contiguous()).contiguous()
     ell = torch.empty((n_t, B), dtype=torch.float32, device=dev)
     coef = torch.empty((n_t, B), dtype=torch.float32, device=dev)

@@ -45,7 +45,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_names(L, bg):
-    assert L.bgpo_abi_version() == 1
+    assert L.bgpo_abi_version() == 2
     assert L.bgpo_status_string(0) == b"BGPO_OK"
     assert L.bgpo_status_string(8) == b"BGPO_ERR_TIMEOUT"
     assert bg.kernel_name(2) == "lmhead_fwd_lse"
@@ -53,10 +53,12 @@ def test_abi_version_and_names(L, bg):
 
 
 def test_problem_struct_layout(bg):
-    assert ctypes.sizeof(bg.BgpoProblem) == 64
+    assert ctypes.sizeof(bg.BgpoProblem) == 72
     assert bg.BgpoProblem.seed.offset == 32
     assert bg.BgpoProblem.trace.offset == 48
     assert bg.BgpoProblem.resp_len.offset == 56
+    assert bg.BgpoProblem.flags.offset == 64
+    assert bg.BgpoProblem.reserved.offset == 68
 
 
 def _prob(bg, **kw):
@@ -87,6 +89,29 @@ def test_validation_rejects_bad_offset_and_nonfinite_scale(L, bg):
     assert L.bgpo_validate_problem(None) == 1
 
 
+def test_validation_of_flags(L, bg):
+    p = _prob(bg)
+    p.flags = bg.FLAG_RECOMPUTE_LOGITS
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 0
+    p.flags = 2                      # unknown bit
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
+    p.flags = 0
+    p.reserved = 7
+    assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+
+
+def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
+    # the kept fp32 logits take 4 * roundup(B R, 256) * roundup(V, 64) bytes
+    # (rounded to the 1 KB region alignment), appended after every other region
+    for (B, R, V) in ((2, 32, 512), (3, 301, 1000), (16, 512, 126464)):
+        keep = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V)))
+        lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, recompute_logits=True)))
+        m_pad = -(-B * R // 256) * 256
+        v_pad = -(-V // 64) * 64
+        assert keep - lean == -(-4 * m_pad * v_pad // 1024) * 1024
+
+
 def test_workspace_independent_of_n_t(L, bg):
     sizes = {n: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, n_t=n))) for n in (1, 2, 16, 32, 1000)}
     assert len(set(sizes.values())) == 1 and sizes[1] > 0
@@ -102,7 +127,11 @@ def test_workspace_of_paper_shapes_fits_hbm(L, bg):
     # LLaDA-8B head, 16 x 512 responses; Dream-7B head, 32 x 1024 (bytes, not n_t-dependent)
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3)
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
+    p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, recompute_logits=True)
+    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 3e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5)
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 40e9
+    p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5, recompute_logits=True)
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 16e9
 
 

@@ -271,9 +271,60 @@ def test_trace_records_every_kernel(bg):
     bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
     names = [n for n, ms in tr.records()]
     assert names == ["mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
-                     "bound_coeffs", "lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
+                     "bound_coeffs", "dz_from_logits", "dx_gemm", "dx_reduce", "dw_gemm"]
     assert all(ms >= 0 for _, ms in tr.records())
     tr.close()
+    # with BGPO_FLAG_RECOMPUTE_LOGITS the backward recomputes the logits on the tensor cores
+    tr = bg.Trace(64)
+    p = bg.problem_from(wl, trace=tr, recompute_logits=True)
+    bg.sample_mask(p, 0, ws)
+    bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    assert [n for n, ms in tr.records()][-4:] == ["lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
+    assert bg.get_device_error(ws) == (0, 0)
+    tr.close()
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged", "ragged_strat"])
+def test_kept_and_recomputed_logits_give_identical_bits(bg, runs, name):
+    # the forward's kept fp32 logits equal the backward GEMM's recomputed ones
+    # (same tiles, same K order) and dz is formed by the same arithmetic, so the
+    # two modes agree bit for bit; both agree with the oracle (test above)
+    import torch
+    wl, inp, g, _ = runs[name]
+    r = gpu_run(wl, inp, recompute_logits=True)
+    assert torch.equal(r["ell"], g["ell"])
+    assert torch.equal(r["dW"], g["dW"])
+    assert torch.equal(r["dX"], g["dX"])
+    assert bg.get_device_error(r["ws"]) == (0, 0) and bg.get_device_error(g["ws"]) == (0, 0)
+
+
+def test_backward_without_kept_logits_is_refused(bg):
+    # the last forward of the sample kept no logits: the backward records
+    # BGPO_ERR_INVALID_ARG and leaves dX and dW untouched
+    import torch
+    wl, inp = _inputs("ragged")
+    keep = bg.problem_from(wl)
+    lean = bg.problem_from(wl, recompute_logits=True)
+    ws = bg.alloc_workspace(keep)
+    ell = torch.empty(wl.B, device="cuda")
+    coef = torch.full((wl.B,), -0.5, device="cuda")
+    dX = torch.zeros((wl.B, wl.R, wl.H), device="cuda")
+    dW = torch.zeros((wl.V, wl.H), device="cuda")
+    bg.sample_mask(keep, 1, ws)
+    bg.elbo_fwd(keep, 1, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_fwd(lean, 1, inp["X"], inp["W"], inp["Y"], ws, ell)     # overrides: no logits kept
+    bg.elbo_bwd_accumulate(keep, 1, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    code, where = bg.get_device_error(ws)
+    assert code == 1 and where == 13 * 16 + 2
+    assert float(dX.abs().max()) == 0.0 and float(dW.abs().max()) == 0.0
+    # a fresh sample that keeps its logits runs normally again
+    bg.clear_device_error(ws)
+    bg.sample_mask(keep, 2, ws)
+    bg.elbo_fwd(keep, 2, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_bwd_accumulate(keep, 2, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    assert bg.get_device_error(ws) == (0, 0)
+    assert float(dW.abs().max()) > 0.0
 
 
 def test_sequence_shards_reproduce_the_full_batch(bg):
