@@ -14,6 +14,8 @@ host<->device copies inside the timed region; `roofline` = the dominant kernel's
 algorithmic tensor FLOP/s against the measured bf16 peak; `cpu_baseline` = the
 fp64 oracle on a bounded sample of the same workload on the host cores.
 `--impl reference` times that oracle alone (the reference arm of this tier).
+`keep_logits` = the same step with BGPO_FLAG_KEEP_LOGITS (the forward keeps its
+fp32 logits, the backward reads them instead of recomputing them).
 """
 import argparse
 import hashlib
@@ -54,6 +56,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-keep-logits", action="store_true",
+                    help="skip the second timed leg with BGPO_FLAG_KEEP_LOGITS")
     ap.add_argument("--grad-variance", action="store_true",
                     help="run the Sec. 4.3 gradient std / bias vs n_t study instead")
     return ap.parse_args()
@@ -285,14 +289,13 @@ def main():
     else:
         bg.group_advantage(prob, inp["rewards"], A)
 
-    # old-policy pass (outside the timed step, forward only, keeps no logits):
-    # l_old on the same draws (Eq. 10)
-    prob_old = bg.problem_from(wl, b_offset=b_offset, recompute_logits=True)
+    # old-policy pass (outside the timed step, forward only): l_old on the same
+    # draws (Eq. 10)
     ell_old = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
     masks = torch.empty((n_t, Bsz, wl.R), dtype=torch.uint8, device=dev)
     for j in range(n_t):
-        bg.sample_mask(prob_old, j, ws, None, masks[j])
-        bg.elbo_fwd(prob_old, j, X, W, Y, ws, ell_old[j])
+        bg.sample_mask(prob, j, ws, None, masks[j])
+        bg.elbo_fwd(prob, j, X, W, Y, ws, ell_old[j])
     ell_old += inp["eps"].T.to(dev)
     masked_per_step = int(masks.sum().item())
     rows_per_sample = masks.reshape(n_t, -1).sum(dim=1).tolist()
@@ -303,84 +306,91 @@ def main():
     dX = torch.zeros((Bsz, wl.R, wl.H), dtype=torch.float32, device=dev)
     dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
 
-    def step(p, X_, W_, Y_, A_, old_):
-        for j in range(n_t):
-            bg.sample_mask(p, j, ws)
-            bg.elbo_fwd(p, j, X_, W_, Y_, ws, ell[j])
-            bg.bound_coeffs(p, j, ell[j], old_[j], A_, coef[j], g[j], ws)
-            bg.elbo_bwd_accumulate(p, j, X_, W_, Y_, coef[j], ws, dX, dW)
-
     def barrier():
         if world > 1:
             import torch.distributed as dist
             dist.barrier()
 
-    for _ in range(args.warmup):
-        step(prob, X, W, Y, A, ell_old)
-    torch.cuda.synchronize()
+    def timed_leg(keep, ws_, sample_clocks):
+        """W warm-up and K timed steps of one mode; per-kernel times from the trace."""
+        def step(p):
+            for j in range(n_t):
+                bg.sample_mask(p, j, ws_)
+                bg.elbo_fwd(p, j, X, W, Y, ws_, ell[j])
+                bg.bound_coeffs(p, j, ell[j], ell_old[j], A, coef[j], g[j], ws_)
+                bg.elbo_bwd_accumulate(p, j, X, W, Y, coef[j], ws_, dX, dW)
 
-    trace = bg.Trace(args.steps * n_t * 12 + 16)
-    prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset)
-    clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
-    stream = torch.cuda.current_stream()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step(prob_t, X, W, Y, A, ell_old)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    clock_info = clocks.stop()
-    ms, masked_all = aggregate_ranks(e0.elapsed_time(e1) / args.steps, masked_per_step)
-    code, where = bg.get_device_error(ws)
-    if code != 0:
-        raise RuntimeError(f"device error {code} at {where}")
-
-    recs = trace.records()
-    gpu_launches = len(recs)
-    per_kernel = {}
-    for name, kms in recs:
-        d = per_kernel.setdefault(name, [0, 0.0])
-        d[0] += 1
-        d[1] += kms
-    trace.close()
+        for _ in range(args.warmup):
+            step(bg.problem_from(wl, b_offset=b_offset, keep_logits=keep))
+        torch.cuda.synchronize()
+        trace = bg.Trace(args.steps * n_t * 12 + 16)
+        prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset, keep_logits=keep)
+        clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+        stream = torch.cuda.current_stream()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        torch.cuda.synchronize()
+        if sample_clocks:
+            clocks.start()
+            time.sleep(0.3)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step(prob_t)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        clock_info = clocks.stop() if sample_clocks else None
+        code, where = bg.get_device_error(ws_)
+        if code != 0:
+            raise RuntimeError(f"device error {code} at {where}")
+        recs = trace.records()
+        per_kernel = {}
+        for name, kms in recs:
+            d = per_kernel.setdefault(name, [0, 0.0])
+            d[0] += 1
+            d[1] += kms
+        trace.close()
+        return e0.elapsed_time(e1) / args.steps, per_kernel, clock_info, len(recs)
 
     peaks = load_peaks()
     H, V = wl.H, wl.V
     gemm_flops_per_step = 2.0 * H * V * masked_per_step   # each GEMM kind of the step
-    gemm_kernels = [k for k in ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
-                    if k in per_kernel]
-    dom = max(gemm_kernels, key=lambda k: per_kernel[k][1])
-    dom_launches, dom_ms = per_kernel[dom]
-    dom_flops_per_launch = gemm_flops_per_step * args.steps / dom_launches
-    dom_avg_s = dom_ms / dom_launches / 1e3
-    achieved = dom_flops_per_launch / dom_avg_s / 1e12
-    traffic = None
-    if dom in TRAFFIC and TRAFFIC[dom]["sha"] == kernel_sha():
-        traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * masked_per_step / n_t
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
+
+    def rooflines(per_kernel):
+        """Dominant GEMM against the sustained bf16 peak; the dz pass (if any) against HBM."""
+        gemm_kernels = [k for k in ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
+                        if k in per_kernel]
+        dom = max(gemm_kernels, key=lambda k: per_kernel[k][1])
+        dom_launches, dom_ms = per_kernel[dom]
+        dom_flops_per_launch = gemm_flops_per_step * args.steps / dom_launches
+        dom_avg_s = dom_ms / dom_launches / 1e3
+        achieved = dom_flops_per_launch / dom_avg_s / 1e12
+        traffic = None
+        if dom in TRAFFIC and TRAFFIC[dom]["sha"] == kernel_sha():
+            traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * masked_per_step / n_t
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
                 "flops_per_launch": dom_flops_per_launch, "avg_launch_ms": dom_avg_s * 1e3}
+        # dL/dz from kept logits: reads 4 V and writes 2 V bytes per masked row
+        hbm_pass = None
+        if "dz_from_logits" in per_kernel:
+            n_dz, dz_ms = per_kernel["dz_from_logits"]
+            dz_bytes = 6.0 * V * masked_per_step * args.steps / n_dz
+            dz_gbs = dz_bytes / (dz_ms / n_dz / 1e3) / 1e9
+            hbm_pass = {"kernel": "dz_from_logits", "bound": "hbm", "achieved": dz_gbs,
+                        "peak": peaks["hbm"], "unit": "GB/s", "frac": dz_gbs / peaks["hbm"],
+                        "bytes_per_launch": dz_bytes, "avg_launch_ms": dz_ms / n_dz,
+                        "peak_kind": f"HBM copy ({peaks['source']})"}
+        return roof, hbm_pass, len(gemm_kernels)
 
-    # dL/dz from the kept logits: reads 4 V and writes 2 V bytes per masked row
-    hbm_pass = None
-    if "dz_from_logits" in per_kernel:
-        n_dz, dz_ms = per_kernel["dz_from_logits"]
-        dz_bytes = 6.0 * V * masked_per_step * args.steps / n_dz
-        dz_gbs = dz_bytes / (dz_ms / n_dz / 1e3) / 1e9
-        hbm_pass = {"kernel": "dz_from_logits", "bound": "hbm", "achieved": dz_gbs,
-                    "peak": peaks["hbm"], "unit": "GB/s", "frac": dz_gbs / peaks["hbm"],
-                    "bytes_per_launch": dz_bytes, "avg_launch_ms": dz_ms / n_dz,
-                    "peak_kind": f"HBM copy ({peaks['source']})"}
-
+    # headline: the default mode (logits recomputed in the backward, never stored)
+    ms_local, per_kernel, clock_info, gpu_launches = timed_leg(False, ws, True)
+    ms, masked_all = aggregate_ranks(ms_local, masked_per_step)
+    roofline, _, n_gemm = rooflines(per_kernel)
     value = masked_all / (ms / 1e3)
-    exec_tflops = len(gemm_kernels) * gemm_flops_per_step / (ms / 1e3) / 1e12
+    exec_tflops = n_gemm * gemm_flops_per_step / (ms / 1e3) / 1e12
     useful_tflops = 3 * gemm_flops_per_step / (ms / 1e3) / 1e12   # fwd, dX, dW
 
     out = {
@@ -388,8 +398,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; shapes of the paper's "
         "LLaDA-8B head, response 512, n_t=16)", "config": config_of(wl),
-        "roofline": roofline, "roofline_hbm_pass": hbm_pass, "gpu_launches": gpu_launches,
-        "clocks": clock_info,
+        "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clock_info,
         "mc_samples_per_s": Bsz * n_t * world / (ms / 1e3),
         "masked_rows_per_step": masked_per_step, "masked_rows_per_sample": rows_per_sample,
         "step_tensor_tflops_executed": exec_tflops,
@@ -399,12 +408,36 @@ def main():
         "peak_mem_bytes": torch.cuda.max_memory_allocated(dev),
         "workspace_bytes": ws.numel(),
     }
-
     if rank == 0:
-        print(f"[bench] {ms:.2f} ms/step, {value:.4g} tok/s, dominant {dom} "
-              f"{achieved:.1f} TFLOP/s, per kernel ms/step: "
+        print(f"[bench] {ms:.2f} ms/step, {value:.4g} tok/s, dominant {roofline['kernel']} "
+              f"{roofline['achieved']:.1f} TFLOP/s, per kernel ms/step: "
               f"{ {k: round(v[1] / args.steps, 3) for k, v in per_kernel.items()} }",
               file=sys.stderr, flush=True)
+
+    # the same step with BGPO_FLAG_KEEP_LOGITS (the forward keeps its fp32 logits,
+    # the backward forms dL/dz from them in one HBM pass instead of a fourth GEMM)
+    if rank == 0 and world == 1 and not args.no_keep_logits:
+        del ws
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats(dev)
+        ws_keep = bg.alloc_workspace(bg.problem_from(wl, b_offset=b_offset, keep_logits=True), dev)
+        k_ms, k_per_kernel, _, k_launches = timed_leg(True, ws_keep, False)
+        k_roof, k_hbm, _ = rooflines(k_per_kernel)
+        out["keep_logits"] = {
+            "value": masked_per_step / (k_ms / 1e3), "unit": UNIT, "ms_per_step": k_ms,
+            "gpu_launches": k_launches, "roofline": k_roof, "roofline_hbm_pass": k_hbm,
+            "step_frac_of_bf16_peak_executed":
+                3 * gemm_flops_per_step / (k_ms / 1e3) / 1e12 / peaks["bf16"],
+            "per_kernel_ms_per_step": {k: v[1] / args.steps for k, v in k_per_kernel.items()},
+            "peak_mem_bytes": torch.cuda.max_memory_allocated(dev),
+            "workspace_bytes": ws_keep.numel()}
+        print(f"[bench] keep_logits: {k_ms:.2f} ms/step, {masked_per_step / (k_ms / 1e3):.4g} tok/s, "
+              f"per kernel ms/step: "
+              f"{ {k: round(v[1] / args.steps, 3) for k, v in k_per_kernel.items()} }",
+              file=sys.stderr, flush=True)
+        del ws_keep
+        torch.cuda.empty_cache()
+
     if rank == 0 and world == 1 and not args.no_e2e:
         out["e2e"] = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev, b_offset)
     elif rank == 0 and world > 1:
@@ -587,8 +620,7 @@ def nt_sweep(bg, dev):
     BGPO and for the ELBO-based objective it bounds (VRPO, Eq. 7), whose weights
     need every sample's l first: "vrpo_retain" keeps one workspace per sample
     (memory grows with n_t), "vrpo_recompute" runs each sample's forward twice.
-    Every backward reads logits its forward kept (the default mode); the first,
-    forward-only pass of "vrpo_recompute" keeps none."""
+    Every backward recomputes its logits (the default mode)."""
     import torch
     from synth import CONFIGS, SWEEP_NT, make_inputs
     base = CONFIGS["llada8b_sweep"]
@@ -599,7 +631,6 @@ def nt_sweep(bg, dev):
     for n_t in SWEEP_NT:
         wl = base.with_(n_t=n_t)
         prob = bg.problem_from(wl)
-        prob_lean = bg.problem_from(wl, recompute_logits=True)
         A = torch.empty(wl.B, dtype=torch.float32, device=dev)
         bg.group_advantage(prob, rewards, A)
         rows = 0
@@ -632,11 +663,10 @@ def nt_sweep(bg, dev):
                         bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
                         bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
                     return
-                p1 = prob if method == "vrpo_retain" else prob_lean
                 for j in range(n_t):
                     ws = wss[j % n_ws]
-                    bg.sample_mask(p1, j, ws)
-                    bg.elbo_fwd(p1, j, X, W, Y, ws, ell[j])
+                    bg.sample_mask(prob, j, ws)
+                    bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
                 bg.vrpo_coeffs(prob, ell, ell, A, cv, None, wss[0])
                 for j in range(n_t):
                     ws = wss[j % n_ws]

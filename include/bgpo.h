@@ -8,8 +8,7 @@
  *   bgpo_sample_mask          t_{b,j} and the response mask (Sec. 2.1; Eq. 3, 5;
  *                             Algorithm 1, sampling of t and y_t)
  *   bgpo_elbo_fwd             l_{b,j} = (1/t) sum_masked log p(y^i | y_t, x) through
- *                             the LM head (Eq. 4); the masked rows' logits are
- *                             kept in the workspace for the backward
+ *                             the LM head (Eq. 4), full logits never stored
  *   bgpo_bound_coeffs         d_j (Eq. 10), g_j (Eq. 13) and dL_j/dl_j with
  *                             L_j = -loss_scale * g_j (Algorithm 1; Eq. 19)
  *   bgpo_elbo_bwd_accumulate  dX += dL_j/dX, dW += dL_j/dW (Algorithm 1, gradient
@@ -34,8 +33,8 @@
  *  - Alignment: X, W, dX, dW and the workspace must be 16-byte aligned
  *    (workspace: 256-byte). H must be a multiple of 64.
  *  - The workspace carries sample j's draws (t, mask), its compacted masked
- *    rows, forward statistics and (unless BGPO_FLAG_RECOMPUTE_LOGITS is set)
- *    the masked rows' logits from one call to the next, so the calls for
+ *    rows, forward statistics and (with BGPO_FLAG_KEEP_LOGITS) the masked
+ *    rows' logits from one call to the next, so the calls for
  *    one sample must be issued in the order
  *        bgpo_sample_mask -> bgpo_elbo_fwd -> [bgpo_bound_coeffs] ->
  *        bgpo_elbo_bwd_accumulate
@@ -82,16 +81,16 @@ typedef struct bgpo_trace bgpo_trace;
 
 /*
  * flags bits
- *   BGPO_FLAG_RECOMPUTE_LOGITS  bgpo_elbo_fwd keeps no logits; the backward of
- *       that sample recomputes them with a fourth tensor-core GEMM. Without the
- *       flag (the default) the forward writes the fp32 logits z = Xm W^T of the
- *       masked rows into the workspace and the backward forms dL/dz from them
- *       in one HBM-bound pass: same results bit for bit, about a quarter less
- *       tensor-core work per sample, 4 * roundup(B R, 256) * roundup(V, 64)
- *       more workspace bytes. Set it for forward-only passes (the old policy's
- *       l_old) or to save memory.
+ *   BGPO_FLAG_KEEP_LOGITS  bgpo_elbo_fwd also writes the fp32 logits z = Xm W^T
+ *       of the masked rows into the workspace, and the backward of that sample
+ *       forms dL/dz from them in one HBM-bound pass instead of recomputing the
+ *       logits with a fourth tensor-core GEMM. Same results bit for bit, a
+ *       quarter less tensor-core work per sample, and
+ *       4 * roundup(B R, 256) * roundup(V, 64) more workspace bytes. Without
+ *       it (the default) full logits never reach device memory. Leave it off
+ *       for forward-only passes (the old policy's l_old).
  */
-#define BGPO_FLAG_RECOMPUTE_LOGITS 1u
+#define BGPO_FLAG_KEEP_LOGITS 1u
 
 /*
  * Problem description (host struct, read by every call; never stored).
@@ -151,10 +150,10 @@ bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
 
 /*
  * Bytes of device workspace the calls below need for `prob`. Depends on B, R,
- * H, V and BGPO_FLAG_RECOMPUTE_LOGITS only -- never on n_t (Linearity, Sec. 3:
+ * H, V and BGPO_FLAG_KEEP_LOGITS only -- never on n_t (Linearity, Sec. 3:
  * one sample's state at a time). The layout without the logits is a prefix of
- * the layout with them, so a workspace sized without the flag also serves
- * calls made with it. Returns 0 for an invalid problem.
+ * the layout with them, so a workspace sized with the flag also serves calls
+ * made without it. Returns 0 for an invalid problem.
  */
 size_t bgpo_workspace_bytes(const bgpo_problem* prob);
 
@@ -183,9 +182,9 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
  * (no length normalisation; an empty mask gives 0). The masked rows of X are
  * gathered, multiplied by W on the tensor cores (bf16 in, fp32 accumulate)
  * and reduced by an online log-sum-exp per row; the per-row log-sum-exp and
- * log-probabilities stay in the workspace for the backward pass, and so do the
- * fp32 logits of the masked rows unless BGPO_FLAG_RECOMPUTE_LOGITS is set
- * (full logits are never written to caller memory). The result is
+ * log-probabilities stay in the workspace for the backward pass. Full logits
+ * are never written, unless BGPO_FLAG_KEEP_LOGITS asks for the masked rows'
+ * fp32 logits to stay in the workspace. The result is
  * deterministic (fixed reduction order), so recomputing l with unchanged inputs
  * gives bit-identical values (on-policy d_j = 0 exactly, Sec. 3.2).
  *   X      device bf16 [B, P+R, H];  W device bf16 [V, H];  Y device int32 [B, R]
@@ -232,19 +231,18 @@ bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const f
  * Backward pass of L_j = sum_b coef_b * l_{b,j}, accumulated (Algorithm 1,
  * gradient accumulation; Eq. 15-17 give the per-sample gradient weights):
  *   w_r   = coef_b / t_{b,j}                       for masked row r = (b, i)
- *   dz_r  = w_r (onehot(Y[b,i]) - softmax(W x_r))  (bf16; the softmax comes
- *           from the logits bgpo_elbo_fwd kept, or with BGPO_FLAG_RECOMPUTE_LOGITS
- *           from logits recomputed on the tensor cores; the two give identical
- *           bits)
+ *   dz_r  = w_r (onehot(Y[b,i]) - softmax(W x_r))  (bf16; logits recomputed
+ *           on the tensor cores, or with BGPO_FLAG_KEEP_LOGITS read from what
+ *           bgpo_elbo_fwd kept; the two give identical bits)
  *   dX[b, i, :] += W^T dz_r        dW += sum_r dz_r x_r^T
  * coef is an input (normally bgpo_bound_coeffs' output for the same j).
  *   dX device float [B, R, H], dW device float [V, H]: accumulated in place.
  * Deterministic: no atomics, fixed summation order.
  * Requires bgpo_sample_mask(j) and bgpo_elbo_fwd(j) before it on the same
- * workspace, with the same X, W and Y. Without BGPO_FLAG_RECOMPUTE_LOGITS the
- * last bgpo_elbo_fwd of sample j must have kept its logits (been called without
- * the flag); otherwise the device error word is set to BGPO_ERR_INVALID_ARG and
- * dX and dW are left unchanged.
+ * workspace, with the same X, W and Y. With BGPO_FLAG_KEEP_LOGITS the last
+ * bgpo_elbo_fwd of sample j must have kept its logits (been called with the
+ * flag too); otherwise the device error word is set to BGPO_ERR_INVALID_ARG
+ * and dX and dW are left unchanged.
  */
 bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
                                      const void* W, const int32_t* Y, const float* coef, void* ws,

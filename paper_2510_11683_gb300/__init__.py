@@ -18,7 +18,7 @@ from ._lib import BgpoError, BgpoProblem  # noqa: F401
 
 T_IID = 0
 T_STRATIFIED = 1
-FLAG_RECOMPUTE_LOGITS = 1   # BGPO_FLAG_RECOMPUTE_LOGITS
+FLAG_KEEP_LOGITS = 1   # BGPO_FLAG_KEEP_LOGITS
 
 
 def _torch():
@@ -27,15 +27,16 @@ def _torch():
 
 
 def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None,
-            b_offset=0, resp_len=None, recompute_logits=False):
+            b_offset=0, resp_len=None, keep_logits=False):
     """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1).
 
     b_offset: global index of the first sequence (a data-parallel shard of a
     larger batch draws the same t and masks as the whole batch would).
     resp_len: optional int32 CUDA tensor [B] of real response lengths (padding
     positions are never masked); the tensor must outlive the calls.
-    recompute_logits: sets BGPO_FLAG_RECOMPUTE_LOGITS (the forward keeps no
-    logits, the backward recomputes them; smaller workspace)."""
+    keep_logits: sets BGPO_FLAG_KEEP_LOGITS (the forward keeps the masked
+    rows' fp32 logits in the workspace and the backward reads them instead of
+    recomputing them; larger workspace, same results)."""
     p = BgpoProblem()
     p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
     p.seed = seed
@@ -43,17 +44,17 @@ def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=
     p.b_offset = b_offset
     p.resp_len = _ptr(resp_len, _torch().int32, "resp_len") if resp_len is not None else None
     p.trace = trace.handle if isinstance(trace, Trace) else trace
-    p.flags = FLAG_RECOMPUTE_LOGITS if recompute_logits else 0
+    p.flags = FLAG_KEEP_LOGITS if keep_logits else 0
     p.reserved = 0
     return p
 
 
 def problem_from(wl, trace=None, loss_scale=None, b_offset=0, resp_len=None,
-                 recompute_logits=False):
+                 keep_logits=False):
     """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
     return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
                    loss_scale=loss_scale, trace=trace, b_offset=b_offset, resp_len=resp_len,
-                   recompute_logits=recompute_logits)
+                   keep_logits=keep_logits)
 
 
 def validate_problem(prob):

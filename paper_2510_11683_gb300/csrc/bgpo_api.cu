@@ -55,7 +55,7 @@ bgpo_status check_problem(const bgpo_problem* p) {
   if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
   if (p->b_offset < 0) return BGPO_ERR_INVALID_ARG;
   if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
-  if ((p->flags & ~BGPO_FLAG_RECOMPUTE_LOGITS) != 0u || p->reserved != 0) return BGPO_ERR_INVALID_ARG;
+  if ((p->flags & ~BGPO_FLAG_KEEP_LOGITS) != 0u || p->reserved != 0) return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
   if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
@@ -67,7 +67,7 @@ bgpo_status check_problem(const bgpo_problem* p) {
 
 Geometry geometry_of(const bgpo_problem* p) { return make_geometry(p->B, p->P, p->R, p->H, p->V); }
 
-bool keeps_logits(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_RECOMPUTE_LOGITS) == 0u; }
+bool keeps_logits(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_KEEP_LOGITS) != 0u; }
 
 bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
   return (j >= 0 && j < p->n_t) ? BGPO_OK : BGPO_ERR_INVALID_ARG;

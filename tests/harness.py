@@ -43,12 +43,12 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None):
 
 
 def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None,
-            recompute_logits=False):
+            keep_logits=False):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
-    The old-policy pass is forward-only and always runs with
-    BGPO_FLAG_RECOMPUTE_LOGITS (it keeps no logits, on the same workspace);
-    `recompute_logits` selects the mode of the inner loop.
+    The old-policy pass is forward-only and keeps no logits; `keep_logits`
+    sets BGPO_FLAG_KEEP_LOGITS for the inner loop (the workspace is sized for
+    it, and the old-policy pass runs on the same workspace without the flag).
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
     masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
@@ -60,9 +60,9 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     if resp_len is not None:
         lens = torch.as_tensor(np.asarray(resp_len), dtype=torch.int32, device=dev)
     prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                           resp_len=lens, recompute_logits=recompute_logits)
+                           resp_len=lens, keep_logits=keep_logits)
     prob_old = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                               resp_len=lens, recompute_logits=True)
+                               resp_len=lens)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     B, n_t = wl.B, wl.n_t

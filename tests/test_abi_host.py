@@ -91,7 +91,7 @@ def test_validation_rejects_bad_offset_and_nonfinite_scale(L, bg):
 
 def test_validation_of_flags(L, bg):
     p = _prob(bg)
-    p.flags = bg.FLAG_RECOMPUTE_LOGITS
+    p.flags = bg.FLAG_KEEP_LOGITS
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 0
     p.flags = 2                      # unknown bit
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
@@ -105,8 +105,8 @@ def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
     # the kept fp32 logits take 4 * roundup(B R, 256) * roundup(V, 64) bytes
     # (rounded to the 1 KB region alignment), appended after every other region
     for (B, R, V) in ((2, 32, 512), (3, 301, 1000), (16, 512, 126464)):
-        keep = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V)))
-        lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, recompute_logits=True)))
+        keep = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, keep_logits=True)))
+        lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V)))
         m_pad = -(-B * R // 256) * 256
         v_pad = -(-V // 64) * 64
         assert keep - lean == -(-4 * m_pad * v_pad // 1024) * 1024
@@ -126,13 +126,13 @@ def test_workspace_grows_with_rows_and_vocab(L, bg):
 def test_workspace_of_paper_shapes_fits_hbm(L, bg):
     # LLaDA-8B head, 16 x 512 responses; Dream-7B head, 32 x 1024 (bytes, not n_t-dependent)
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3)
-    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
-    p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, recompute_logits=True)
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 3e9
+    p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, keep_logits=True)
+    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5)
-    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 40e9
-    p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5, recompute_logits=True)
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 16e9
+    p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5, keep_logits=True)
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 40e9
 
 
 FAKE = 1 << 20  # an aligned, never dereferenced address

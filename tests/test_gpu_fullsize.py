@@ -112,3 +112,17 @@ def test_full_head_complete_dw_parity(bg):
     assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= 1e-3
     assert normwise(to64(g["dW"]), o["dW"]) <= 2e-2
     assert normwise(to64(g["dX"]), o["dX"]) <= 2e-2
+
+
+def test_keep_logits_bit_identical_at_full_head(bg):
+    # BGPO_FLAG_KEEP_LOGITS reads back the forward's fp32 logits instead of
+    # recomputing them: same l, dX and dW bits at the full LLaDA-8B head
+    import torch
+    wl = CONFIGS["llada8b_r256"]
+    inp = make_inputs(wl, device="cuda")
+    a = gpu_run(wl, inp)
+    b = gpu_run(wl, inp, keep_logits=True)
+    assert bg.get_device_error(a["ws"]) == (0, 0) and bg.get_device_error(b["ws"]) == (0, 0)
+    assert torch.equal(a["ell"], b["ell"])
+    assert torch.equal(a["dX"], b["dX"])
+    assert torch.equal(a["dW"], b["dW"])

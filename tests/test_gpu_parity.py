@@ -271,16 +271,17 @@ def test_trace_records_every_kernel(bg):
     bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
     names = [n for n, ms in tr.records()]
     assert names == ["mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
-                     "bound_coeffs", "dz_from_logits", "dx_gemm", "dx_reduce", "dw_gemm"]
+                     "bound_coeffs", "lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
     assert all(ms >= 0 for _, ms in tr.records())
     tr.close()
-    # with BGPO_FLAG_RECOMPUTE_LOGITS the backward recomputes the logits on the tensor cores
+    # with BGPO_FLAG_KEEP_LOGITS the backward reads the logits the forward kept
     tr = bg.Trace(64)
-    p = bg.problem_from(wl, trace=tr, recompute_logits=True)
+    p = bg.problem_from(wl, trace=tr, keep_logits=True)
+    ws = bg.alloc_workspace(p)
     bg.sample_mask(p, 0, ws)
     bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
     bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
-    assert [n for n, ms in tr.records()][-4:] == ["lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
+    assert [n for n, ms in tr.records()][-4:] == ["dz_from_logits", "dx_gemm", "dx_reduce", "dw_gemm"]
     assert bg.get_device_error(ws) == (0, 0)
     tr.close()
 
@@ -292,7 +293,7 @@ def test_kept_and_recomputed_logits_give_identical_bits(bg, runs, name):
     # two modes agree bit for bit; both agree with the oracle (test above)
     import torch
     wl, inp, g, _ = runs[name]
-    r = gpu_run(wl, inp, recompute_logits=True)
+    r = gpu_run(wl, inp, keep_logits=True)
     assert torch.equal(r["ell"], g["ell"])
     assert torch.equal(r["dW"], g["dW"])
     assert torch.equal(r["dX"], g["dX"])
@@ -304,8 +305,8 @@ def test_backward_without_kept_logits_is_refused(bg):
     # BGPO_ERR_INVALID_ARG and leaves dX and dW untouched
     import torch
     wl, inp = _inputs("ragged")
-    keep = bg.problem_from(wl)
-    lean = bg.problem_from(wl, recompute_logits=True)
+    keep = bg.problem_from(wl, keep_logits=True)
+    lean = bg.problem_from(wl)
     ws = bg.alloc_workspace(keep)
     ell = torch.empty(wl.B, device="cuda")
     coef = torch.full((wl.B,), -0.5, device="cuda")
