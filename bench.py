@@ -41,8 +41,8 @@ UNIT = "tokens/s"
 # masked rows M (the dW read-modify-write is fixed, dZ / Xm reads grow with M).
 # Valid only while the GEMM sources hash to `sha`.
 TRAFFIC = {
-    "dw_gemm": {"fixed_bytes": 4.0309e+09, "bytes_per_row": 336850.9,
-                "sha": "3247d9acaa21ce7a4788fe5fa143b0b633c39a0b72720e298c89d2d9d22f6888"},
+    "dw_gemm": {"fixed_bytes": 4.0171e+09, "bytes_per_row": 353320.7,
+                "sha": "ef1569afb7fba77960e8ba13e1584f385ab49ab995479888074c54fcde49e576"},
 }
 
 

@@ -326,6 +326,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   ga.j = j;
   ga.coef = coef;
   ga.dW = dW;
+  ga.dX = dX;
   if (keep) {
     TraceScope ts(prob->trace, KID_DZ_FROM_LOGITS, s);
     if (launch_dz_from_logits(g, j, coef, sms, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
@@ -341,7 +342,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   }
   {
     TraceScope ts(prob->trace, KID_DX_REDUCE, s);
-    if (launch_dx_reduce(g, j, ga.num_pairs, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_dx_reduce(g, j, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
   {
     TraceScope ts(prob->trace, KID_DW_GEMM, s);

@@ -52,8 +52,8 @@ cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, flo
 cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
                                 const float* ell_old, const float* A, float* coef_out,
                                 float* g_out, const WsPtrs& w, cudaStream_t s);
-cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_pairs, const WsPtrs& w,
-                             float* dX, cudaStream_t s);
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* dX,
+                             cudaStream_t s);
 cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
                                    cudaStream_t s);
 cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
@@ -70,6 +70,7 @@ struct GemmArgs {
   int32_t j;
   const float* coef;  // GEMM_DZ: per-sequence dL/dl
   float* dW;          // GEMM_DW: accumulated weight gradient [V, H]
+  float* dX = nullptr;  // GEMM_DX: accumulated dHidden [B, R, H] (written directly without split-K)
 };
 
 // CTA pairs the GEMM kernels run as: the 2-CTA clusters that fit on the

@@ -106,7 +106,8 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
 // Device workspace layout. Every region starts on a 1024-byte boundary (TMA
 // tiles with 128-byte swizzle want 1024-byte aligned bases).
 struct WsLayout {
-  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M, [4] logits kept
+  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M, [4] logits kept,
+                     //            [5] dX split count
   size_t t;          // float[B]    t_{b,j}
   size_t tnum;       // uint32[2B]  T numerator (t = T / D), (low, high) words
   size_t seg_off;    // int32[B+1]  first compacted row of each sequence
@@ -163,6 +164,9 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
 // Indices into the int32 error word. ERR_LOGITS is 1 while the logit region
 // holds the current sample's logits (set by the forward that wrote them,
 // cleared by the masking of a new sample and by a forward that keeps none).
-enum ErrField : int { ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4 };
+// ERR_DX_SPLITS is the split-K count the last dX GEMM used.
+enum ErrField : int {
+  ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4, ERR_DX_SPLITS = 5
+};
 
 }  // namespace bgpo

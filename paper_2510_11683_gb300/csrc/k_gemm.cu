@@ -24,7 +24,8 @@
 //   GEMM_DZ   z = Xm W^T recomputed (when the forward kept no logits);
 //             epilogue: dz = w_r (onehot - e^{z - lse}) stored as bf16
 //             (gradient of Eq. 4 weighted by Eq. 13's dL/dl).
-//   GEMM_DX   dXm = dZ W (K = vocabulary, split-K partials in fp32).
+//   GEMM_DX   dXm = dZ W (K = vocabulary): split-K partials in fp32, or, when
+//             the launch needs no split, added straight into the dX rows.
 //   GEMM_DW   dW += dZ^T Xm (K = masked rows), fp32 TMA reduce-add.
 //
 // Every wait is bounded (time and polls); a wait that runs out sets the
@@ -55,6 +56,7 @@ struct GemmParams {
   WsPtrs w;
   const float* coef;
   float* dW;
+  float* dX;
 };
 
 struct Work {
@@ -346,17 +348,39 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
 
 // GEMM_DX: fp32 partial of split s, rows [split * tiles_m * 256 + r] of the
 // partial buffer, 32-column sub-tiles through TMA stores (rows >= M hold zeros).
-__device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* map_c,
+// Without split-K every dX element has exactly this one contribution in the
+// launch, so the lane adds its row's sub-tile straight into dX[b, i] (the row
+// the compaction recorded), 128 contiguous bytes per sub-tile, and the split
+// reduction after the GEMM has nothing to do.
+__device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
                                        const Work& wk, const Unit& t, int64_t row0, int lane,
                                        uint32_t tb, EpiStage& st) {
   const int32_t h0 = t.n_blk * kBN;
   const int32_t prow0 = (int32_t)(t.split * wk.tiles_m * kPairM + row0);
+  const int64_t r = row0 + lane;
+  float4* drow = nullptr;
+  if (wk.splits == 1 && r < M)
+    drow = reinterpret_cast<float4*>(p.dX + (int64_t)p.w.rows[r] * p.g.H + h0);
 #pragma unroll 1
   for (int c = 0; c < kBN / 32; ++c) {
     if (h0 + c * 32 >= p.g.H) break;  // warp-uniform
     uint32_t raw[32];
     tmem_ld_32x32b_x32(tb + c * 32, raw);
     tmem_ld_wait();
+    if (wk.splits == 1) {  // launch-uniform
+      if (drow) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          float4 o = drow[c * 8 + q];
+          o.x += bits_f(raw[4 * q]);
+          o.y += bits_f(raw[4 * q + 1]);
+          o.z += bits_f(raw[4 * q + 2]);
+          o.w += bits_f(raw[4 * q + 3]);
+          drow[c * 8 + q] = o;
+        }
+      }
+      continue;
+    }
     uint4 chunk[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q)
@@ -441,6 +465,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     set_device_error(err, kStatusInvalidArg, kernel_id<KIND>() * 16 + 1);
   }
   const Work wk = make_work<KIND>(p, M);
+  // the split reduction after the dX GEMM reads the split count from here
+  if (KIND == GEMM_DX && blockIdx.x == 0 && threadIdx.x == 0) err[ERR_DX_SPLITS] = wk.splits;
   if (pair >= wk.units) return;  // both CTAs of the pair, before any allocation
 
   if (threadIdx.x == 0) {
@@ -573,7 +599,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int64_t row0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM + quarter * 32;
       if (KIND == GEMM_FWD) epi_fwd(p, &map_c, M, t, row0, lane, tb, st);
       else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, lane, tb, st);
-      else if (KIND == GEMM_DX) epi_dx(p, &map_c, wk, t, row0, lane, tb, st);
+      else if (KIND == GEMM_DX) epi_dx(p, &map_c, M, wk, t, row0, lane, tb, st);
       else epi_dw(p, &map_c, t, row0, lane, tb, st);
       tc_fence_before();
       __syncwarp();
@@ -640,6 +666,7 @@ cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorM
   p.w = w;
   p.coef = a.coef;
   p.dW = a.dW;
+  p.dX = a.dX;
   switch (kind) {
     case GEMM_FWD: return launch_kind<GEMM_FWD>(map_a, map_b, map_c, p, s);
     case GEMM_DZ: return launch_kind<GEMM_DZ>(map_a, map_b, map_c, p, s);

@@ -331,15 +331,21 @@ __global__ void k_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const fl
 
 // ---------------------------------------------------------------------------
 // dX[b, i, :] += sum_s partial_s[r, :] over the split-K partials of the dX GEMM
-// (fixed split order; rows are unique within a sample, so no atomics).
+// (fixed split order; rows are unique within a sample, so no atomics). With a
+// single split the GEMM's epilogue has already added its tile into dX.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, int num_pairs, WsPtrs w,
+__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs w,
                                                    float* __restrict__ dX) {
   const int32_t M = rows_of_sample(w.err, j, KID_DX_REDUCE);
   const int64_t r = blockIdx.x;
   if (r >= M) return;
   const int64_t mb = ceil_div(M, kPairM);
-  const int S = dx_splits(mb, g.tiles_h, num_pairs, g.kb_v, dxp_row_block_cap(g));
+  const int S = w.err[ERR_DX_SPLITS];  // written by the dX GEMM of this sample
+  if (S == 1) return;
+  if (S < 1 || S > kMaxSplits || S * mb > dxp_row_block_cap(g)) {  // not a count it can write
+    if (r == 0 && threadIdx.x == 0) set_device_error(w.err, kStatusInvalidArg, KID_DX_REDUCE * 16 + 2);
+    return;
+  }
   const int64_t split_stride = mb * kPairM * g.H / 4;
   const float4* src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
   float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)w.rows[r] * (g.H / 4);
@@ -469,9 +475,9 @@ cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const f
   return cudaGetLastError();
 }
 
-cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, int num_pairs, const WsPtrs& w, float* dX,
+cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* dX,
                              cudaStream_t s) {
-  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, num_pairs, w, dX);
+  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, w, dX);
   return cudaGetLastError();
 }
 
