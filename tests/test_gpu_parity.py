@@ -389,3 +389,50 @@ def test_variable_length_responses(bg):
     assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL
     assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL
     assert float(g["dX"][2, 117:].abs().max()) == 0.0
+
+
+@pytest.mark.parametrize("keep", [False, True])
+def test_whole_step_replays_from_a_cuda_graph(bg, keep):
+    # the n_t loop allocates nothing, never synchronises and keeps M on the
+    # device, so one step captures into a CUDA graph; a replay gives the bits
+    # of the eager step
+    import torch
+    wl, inp = _inputs("ragged")
+    p = bg.problem_from(wl, keep_logits=keep)
+    X, W, Y = inp["X"], inp["W"], inp["Y"]
+    ws = bg.alloc_workspace(p)
+    A = torch.empty(wl.B, device="cuda")
+    bg.group_advantage(p, inp["rewards"], A)          # ragged draws Bernoulli rewards
+    ell_old = torch.empty((wl.n_t, wl.B), device="cuda")
+    for j in range(wl.n_t):
+        bg.sample_mask(p, j, ws)
+        bg.elbo_fwd(p, j, X, W, Y, ws, ell_old[j])
+    ell_old += inp["eps"].T
+
+    def step(out):
+        for j in range(wl.n_t):
+            bg.sample_mask(p, j, ws)
+            bg.elbo_fwd(p, j, X, W, Y, ws, out["ell"][j])
+            bg.bound_coeffs(p, j, out["ell"][j], ell_old[j], A, out["coef"][j], None, ws)
+            bg.elbo_bwd_accumulate(p, j, X, W, Y, out["coef"][j], ws, out["dX"], out["dW"])
+
+    def buffers():
+        return dict(ell=torch.empty((wl.n_t, wl.B), device="cuda"),
+                    coef=torch.empty((wl.n_t, wl.B), device="cuda"),
+                    dX=torch.zeros((wl.B, wl.R, wl.H), device="cuda"),
+                    dW=torch.zeros((wl.V, wl.H), device="cuda"))
+
+    eager = buffers()
+    step(eager)
+    torch.cuda.synchronize()
+    graphed = buffers()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step(graphed)
+    graphed["dX"].zero_()
+    graphed["dW"].zero_()
+    graph.replay()
+    torch.cuda.synchronize()
+    assert bg.get_device_error(ws) == (0, 0)
+    for k in ("ell", "coef", "dX", "dW"):
+        assert torch.equal(graphed[k], eager[k]), k
