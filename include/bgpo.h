@@ -47,6 +47,12 @@
  *    in an error word inside the workspace: read it with bgpo_get_device_error.
  *  - The device must have compute capability 10.3 (GB300); otherwise every
  *    launching call returns BGPO_ERR_UNSUPPORTED_DEVICE.
+ *  - A checked build of the same library (compiled with -DBGPO_CHECKED) tests
+ *    every index it reads from device memory (masked-row lists, segment
+ *    offsets, row counts, split counts) and every target token against its
+ *    buffer before use; a failed test records BGPO_ERR_BOUNDS in the error word
+ *    and skips the access. It stands in for a memory checker. The normal build
+ *    trusts these values, which its own kernels wrote.
  */
 #ifndef BGPO_H_
 #define BGPO_H_
@@ -69,7 +75,10 @@ typedef enum bgpo_status {
   BGPO_ERR_NONFINITE = 5,            /* non-finite bound coefficient (device) */
   BGPO_ERR_UNSUPPORTED_DEVICE = 6,   /* current device is not sm_103 */
   BGPO_ERR_CUDA = 7,                 /* a CUDA runtime call or launch failed */
-  BGPO_ERR_TIMEOUT = 8               /* a bounded device-side wait ran out */
+  BGPO_ERR_TIMEOUT = 8,              /* a bounded device-side wait ran out */
+  BGPO_ERR_BOUNDS = 9                /* checked build only: an index read from device
+                                        memory fell outside its buffer; the access
+                                        was skipped (device) */
 } bgpo_status;
 
 /* Optional per-kernel timing: CUDA events recorded around each kernel launch. */

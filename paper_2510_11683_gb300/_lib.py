@@ -2,7 +2,7 @@
 import ctypes
 import os
 
-from .build import LIB_PATH
+from .build import CHECKED_LIB_PATH, LIB_PATH
 
 c_int32 = ctypes.c_int32
 c_void_p = ctypes.c_void_p
@@ -12,7 +12,7 @@ BGPO_OK = 0
 STATUS_NAMES = {
     0: "BGPO_OK", 1: "BGPO_ERR_INVALID_ARG", 2: "BGPO_ERR_SHAPE", 3: "BGPO_ERR_ALIGNMENT",
     4: "BGPO_ERR_WORKSPACE_TOO_SMALL", 5: "BGPO_ERR_NONFINITE", 6: "BGPO_ERR_UNSUPPORTED_DEVICE",
-    7: "BGPO_ERR_CUDA", 8: "BGPO_ERR_TIMEOUT",
+    7: "BGPO_ERR_CUDA", 8: "BGPO_ERR_TIMEOUT", 9: "BGPO_ERR_BOUNDS",
 }
 
 
@@ -69,16 +69,26 @@ class BgpoError(RuntimeError):
         super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)}")
 
 
+def lib_path():
+    """lib/libbgpo.so, or with BGPO_LIBRARY=checked in the environment the
+    bounds-checked build lib/libbgpo_checked.so."""
+    choice = os.environ.get("BGPO_LIBRARY", "")
+    if choice not in ("", "checked"):
+        raise ValueError(f"BGPO_LIBRARY must be unset or 'checked', got {choice!r}")
+    return CHECKED_LIB_PATH if choice == "checked" else LIB_PATH
+
+
 def lib():
-    """Loads lib/libbgpo.so (built by build.py); raises if it is missing."""
+    """Loads the library lib_path() names (built by build.py); raises if it is missing."""
     global _LIB
     if _LIB is None:
-        if not os.path.exists(LIB_PATH):
+        path = lib_path()
+        if not os.path.exists(path):
             raise ImportError(
-                f"CUDA library {LIB_PATH} is missing: build it with "
+                f"CUDA library {path} is missing: build it with "
                 "`python -c 'import __graft_entry__ as g; g.build()'` "
-                "or `python -m paper_2510_11683_gb300.build`")
-        h = ctypes.CDLL(LIB_PATH)
+                "or `python -m paper_2510_11683_gb300.build [--checked]`")
+        h = ctypes.CDLL(path)
         for name, (res, args) in SIGNATURES.items():
             f = getattr(h, name)
             f.restype = res

@@ -1,7 +1,9 @@
 """Builds the in-tree CUDA library ``lib/libbgpo.so`` for sm_103a with nvcc.
 
 Translation units are compiled in parallel and linked into one shared library
-(static CUDA runtime). ``python -m paper_2510_11683_gb300.build`` runs it.
+(static CUDA runtime). ``python -m paper_2510_11683_gb300.build`` runs it;
+``--checked`` builds ``lib/libbgpo_checked.so`` instead, the same sources with
+-DBGPO_CHECKED (device-side bounds checks that record BGPO_ERR_BOUNDS).
 """
 import os
 import subprocess
@@ -14,6 +16,7 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB_DIR = os.path.join(PKG_DIR, "lib")
 LIB_PATH = os.path.join(LIB_DIR, "libbgpo.so")
+CHECKED_LIB_PATH = os.path.join(LIB_DIR, "libbgpo_checked.so")
 OBJ_DIR = os.path.join(PKG_DIR, "_build")
 
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -27,8 +30,8 @@ def nvcc():
     return cand if os.path.exists(cand) else "nvcc"
 
 
-def _compile(src, extra, verbose):
-    obj = os.path.join(OBJ_DIR, os.path.splitext(src)[0] + ".o")
+def _compile(src, extra, obj_dir, verbose):
+    obj = os.path.join(obj_dir, os.path.splitext(src)[0] + ".o")
     cmd = [nvcc(), *ARCH_FLAGS, *COMMON_FLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj]
     if verbose:
         print(" ".join(cmd), flush=True)
@@ -40,21 +43,25 @@ def _compile(src, extra, verbose):
     return obj
 
 
-def build(verbose=False, ptxas_verbose=False):
-    """Compiles every CUDA source and links lib/libbgpo.so. Returns its path."""
-    os.makedirs(OBJ_DIR, exist_ok=True)
+def build(verbose=False, ptxas_verbose=False, checked=False):
+    """Compiles every CUDA source and links lib/libbgpo.so (checked=True:
+    lib/libbgpo_checked.so with -DBGPO_CHECKED). Returns its path."""
+    obj_dir = os.path.join(OBJ_DIR, "checked") if checked else OBJ_DIR
+    out = CHECKED_LIB_PATH if checked else LIB_PATH
+    os.makedirs(obj_dir, exist_ok=True)
     os.makedirs(LIB_DIR, exist_ok=True)
-    extra = ["-Xptxas", "-v"] if ptxas_verbose else []
+    extra = (["-Xptxas", "-v"] if ptxas_verbose else []) + (["-DBGPO_CHECKED"] if checked else [])
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(lambda s: _compile(s, extra, verbose or ptxas_verbose), SOURCES))
-    tmp = LIB_PATH + ".tmp"
+        objs = list(ex.map(lambda s: _compile(s, extra, obj_dir, verbose or ptxas_verbose),
+                           SOURCES))
+    tmp = out + ".tmp"
     cmd = [nvcc(), *ARCH_FLAGS, "-shared", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, out)
+    return out
 
 
 if __name__ == "__main__":
-    print(build(verbose=True, ptxas_verbose="-v" in sys.argv))
+    print(build(verbose=True, ptxas_verbose="-v" in sys.argv, checked="--checked" in sys.argv))

@@ -1,10 +1,11 @@
 // Host side of the C ABI declared in include/bgpo.h: argument validation,
-// workspace layout, TMA tensor-map encoding, kernel launches and per-kernel
-// event tracing. Keeps no state between calls except the cached driver entry
+// workspace layout, TMA tensor-map encoding, kernel launches, per-kernel
+// event tracing and an NVTX range named after each launching call. Keeps no state between calls except the cached driver entry
 // point of cuTensorMapEncodeTiled.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -48,6 +49,15 @@ struct TraceScope {
   ~TraceScope() {
     if (idx >= 0) cudaEventRecord(tr->stop[idx], s);
   }
+};
+
+// NVTX range around one launching C-ABI call, named after it (shows in Nsight
+// timelines; a no-op when no tool is attached).
+struct CallRange {
+  explicit CallRange(const char* name) { nvtxRangePushA(name); }
+  ~CallRange() { nvtxRangePop(); }
+  CallRange(const CallRange&) = delete;
+  CallRange& operator=(const CallRange&) = delete;
 };
 
 bgpo_status check_problem(const bgpo_problem* p) {
@@ -156,6 +166,7 @@ const char* bgpo_status_string(bgpo_status s) {
     case BGPO_ERR_UNSUPPORTED_DEVICE: return "BGPO_ERR_UNSUPPORTED_DEVICE";
     case BGPO_ERR_CUDA: return "BGPO_ERR_CUDA";
     case BGPO_ERR_TIMEOUT: return "BGPO_ERR_TIMEOUT";
+    case BGPO_ERR_BOUNDS: return "BGPO_ERR_BOUNDS";
   }
   return "BGPO_ERR_UNKNOWN";
 }
@@ -169,6 +180,7 @@ size_t bgpo_workspace_bytes(const bgpo_problem* prob) {
 
 bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size_t ws_bytes,
                              float* t_out, uint8_t* mask_out, void* stream) {
+  CallRange range("bgpo_sample_mask");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if ((st = check_sample(prob, j)) != BGPO_OK) return st;
@@ -198,6 +210,7 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
 bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, const void* W,
                           const int32_t* Y, void* ws, size_t ws_bytes, float* ell_out,
                           void* stream) {
+  CallRange range("bgpo_elbo_fwd");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if ((st = check_sample(prob, j)) != BGPO_OK) return st;
@@ -249,6 +262,7 @@ bgpo_status bgpo_elbo_fwd(const bgpo_problem* prob, int32_t j, const void* X, co
 bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* ell,
                               const float* ell_old, const float* A, float* coef_out, float* g_out,
                               void* ws, size_t ws_bytes, void* stream) {
+  CallRange range("bgpo_bound_coeffs");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if ((st = check_sample(prob, j)) != BGPO_OK) return st;
@@ -270,6 +284,7 @@ bgpo_status bgpo_bound_coeffs(const bgpo_problem* prob, int32_t j, const float* 
 bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const float* ell_old,
                              const float* A, float* coef_out, float* R_out, void* ws,
                              size_t ws_bytes, void* stream) {
+  CallRange range("bgpo_vrpo_coeffs");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if (!ell || !ell_old || !A || !coef_out) return BGPO_ERR_INVALID_ARG;
@@ -290,6 +305,7 @@ bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const f
 bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const void* X,
                                      const void* W, const int32_t* Y, const float* coef, void* ws,
                                      size_t ws_bytes, float* dX, float* dW, void* stream) {
+  CallRange range("bgpo_elbo_bwd_accumulate");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if ((st = check_sample(prob, j)) != BGPO_OK) return st;
@@ -354,6 +370,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
 
 bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards, float* A_out,
                                  void* stream) {
+  CallRange range("bgpo_group_advantage");
   bgpo_status st = check_problem(prob);
   if (st != BGPO_OK) return st;
   if (!rewards || !A_out) return BGPO_ERR_INVALID_ARG;

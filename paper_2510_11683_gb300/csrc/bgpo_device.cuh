@@ -24,6 +24,17 @@ __device__ __forceinline__ void set_device_error(int32_t* err, int32_t status, i
   if (atomicCAS(&err[ERR_STATUS], 0, status) == 0) atomicExch(&err[ERR_WHERE], where);
 }
 
+// Bounds checks of the checked build (compiled with -DBGPO_CHECKED): a check
+// that fails records BGPO_ERR_BOUNDS (9) and `where` in the workspace error word
+// and evaluates to false, so that the caller skips the guarded access. The
+// normal build does not evaluate the condition.
+#ifdef BGPO_CHECKED
+#define BGPO_IN_BOUNDS(err, cond, where) \
+  ((cond) ? true : (::bgpo::set_device_error((err), 9, (where)), false))
+#else
+#define BGPO_IN_BOUNDS(err, cond, where) true
+#endif
+
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -304,7 +304,8 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
   const bool valid = r < M;
   float w = 0.f, lse_l2 = 0.f;
   int32_t y = -1;
-  if (valid) {
+  if (valid && BGPO_IN_BOUNDS(p.w.err, p.w.rows[r] >= 0 && p.w.rows[r] < p.g.m_cap,
+                              KID_LMHEAD_DZ * 16 + 10)) {
     const int32_t b = p.w.rows[r] / (int32_t)p.g.R;
     w = p.coef[b] / p.w.t[b];
     lse_l2 = p.w.lse[r] * kLog2e;
@@ -359,7 +360,8 @@ __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* m
   const int32_t prow0 = (int32_t)(t.split * wk.tiles_m * kPairM + row0);
   const int64_t r = row0 + lane;
   float4* drow = nullptr;
-  if (wk.splits == 1 && r < M)
+  if (wk.splits == 1 && r < M &&
+      BGPO_IN_BOUNDS(p.w.err, p.w.rows[r] >= 0 && p.w.rows[r] < p.g.m_cap, KID_DX_GEMM * 16 + 10))
     drow = reinterpret_cast<float4*>(p.dX + (int64_t)p.w.rows[r] * p.g.H + h0);
 #pragma unroll 1
   for (int c = 0; c < kBN / 32; ++c) {
@@ -464,6 +466,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   } else if (blockIdx.x == 0 && threadIdx.x == 0) {
     set_device_error(err, kStatusInvalidArg, kernel_id<KIND>() * 16 + 1);
   }
+  if (!BGPO_IN_BOUNDS(err, M >= 0 && M <= p.g.m_cap, kernel_id<KIND>() * 16 + 9)) M = 0;
   const Work wk = make_work<KIND>(p, M);
   // the split reduction after the dX GEMM reads the split count from here
   if (KIND == GEMM_DX && blockIdx.x == 0 && threadIdx.x == 0) err[ERR_DX_SPLITS] = wk.splits;

@@ -105,7 +105,11 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
       int32_t pos = excl;
 #pragma unroll
       for (int k = 0; k < 4; ++k)
-        if ((bits >> k) & 1u) w.rows[pos++] = b * a.R + 4 * q + k;
+        if ((bits >> k) & 1u) {
+          if (BGPO_IN_BOUNDS(w.err, pos < a.B * a.R, KID_MASK_COMPACT * 16 + 9))
+            w.rows[pos] = b * a.R + 4 * q + k;
+          ++pos;
+        }
     }
     __syncthreads();
     if (tid == kScanThreads - 1) s_carry = excl + cnt;
@@ -129,6 +133,7 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
 __global__ void __launch_bounds__(256) k_gather(Geometry g, int32_t j, const uint4* __restrict__ X,
                                                 const int32_t* __restrict__ Y, WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_GATHER);
+  if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_GATHER * 16 + 9)) return;
   const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= round_up(M, kPairM)) return;
@@ -136,10 +141,15 @@ __global__ void __launch_bounds__(256) k_gather(Geometry g, int32_t j, const uin
   uint4* dst = reinterpret_cast<uint4*>(w.xm) + r * nvec;
   if (r < M) {
     const int32_t idx = w.rows[r];
+    if (!BGPO_IN_BOUNDS(w.err, idx >= 0 && idx < g.m_cap, KID_GATHER * 16 + 10)) return;
     const int64_t b = idx / g.R, i = idx % g.R;
     const uint4* src = X + (b * (g.P + g.R) + g.P + i) * nvec;
     for (int64_t v = lane; v < nvec; v += 32) dst[v] = __ldg(src + v);
-    if (lane == 0) w.tgt[r] = __ldg(Y + idx);
+    if (lane == 0) {
+      const int32_t y = __ldg(Y + idx);
+      (void)BGPO_IN_BOUNDS(w.err, y >= 0 && y < g.V, KID_GATHER * 16 + 11);  // a target outside V
+      w.tgt[r] = y;
+    }
   } else {
     const uint4 z = make_uint4(0, 0, 0, 0);
     for (int64_t v = lane; v < nvec; v += 32) dst[v] = z;
@@ -213,6 +223,7 @@ __global__ void __launch_bounds__(kDzThreads, 4)
     }
     return;
   }
+  if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_DZ_FROM_LOGITS * 16 + 9)) return;
   const int64_t nvec = g.v_pad / 8;
   const int64_t per_row = ceil_div(nvec, kDzItemVecs);
   const int64_t items = round_up(M, kPairM) * per_row;
@@ -226,7 +237,9 @@ __global__ void __launch_bounds__(kDzThreads, 4)
     float wr = 0.f, lse_l2 = 0.f;
     int32_t y = -1;
     if (valid) {
-      const int32_t b = w.rows[r] / (int32_t)g.R;
+      const int32_t idx = w.rows[r];
+      if (!BGPO_IN_BOUNDS(w.err, idx >= 0 && idx < g.m_cap, KID_DZ_FROM_LOGITS * 16 + 10)) continue;
+      const int32_t b = idx / (int32_t)g.R;
       wr = coef[b] / w.t[b];
       lse_l2 = w.lse[r] * kLog2e;
       y = w.tgt[r];
@@ -280,7 +293,8 @@ __global__ void __launch_bounds__(256) k_seq_reduce(Geometry g, int32_t j, WsPtr
   float acc = 0.f;
   if (M > 0) {
     const int32_t lo = w.seg_off[b], hi = w.seg_off[b + 1];
-    for (int32_t r = lo + lane; r < hi; r += 32) acc += w.logp[r];
+    if (BGPO_IN_BOUNDS(w.err, 0 <= lo && lo <= hi && hi <= M && M <= g.m_cap, KID_SEQ_REDUCE * 16 + 9))
+      for (int32_t r = lo + lane; r < hi; r += 32) acc += w.logp[r];
   }
   acc = warp_sum(acc);
   if (lane == 0) ell_out[b] = acc / w.t[b];
@@ -347,8 +361,10 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
     return;
   }
   const int64_t split_stride = mb * kPairM * g.H / 4;
+  const int32_t idx = w.rows[r];
+  if (!BGPO_IN_BOUNDS(w.err, idx >= 0 && idx < g.m_cap, KID_DX_REDUCE * 16 + 9)) return;
   const float4* src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
-  float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)w.rows[r] * (g.H / 4);
+  float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)idx * (g.H / 4);
   for (int64_t h = threadIdx.x; h < g.H / 4; h += blockDim.x) {
     float4 acc = src[h];
     for (int s = 1; s < S; ++s) {

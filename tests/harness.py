@@ -6,13 +6,15 @@ import numpy as np
 from oracle import bgpo_oracle as O
 
 
-def ensure_built():
-    """Builds lib/libbgpo.so when it is missing (nvcc cross-compiles without a GPU)."""
+def ensure_built(checked=False):
+    """Builds lib/libbgpo.so (checked=True: lib/libbgpo_checked.so) when it is
+    missing (nvcc cross-compiles without a GPU)."""
     import os
     from paper_2510_11683_gb300 import build as B
-    if not os.path.exists(B.LIB_PATH):
-        B.build()
-    return B.LIB_PATH
+    path = B.CHECKED_LIB_PATH if checked else B.LIB_PATH
+    if not os.path.exists(path):
+        B.build(checked=checked)
+    return path
 
 
 def to64(t):

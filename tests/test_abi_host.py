@@ -48,6 +48,7 @@ def test_abi_version_and_names(L, bg):
     assert L.bgpo_abi_version() == 2
     assert L.bgpo_status_string(0) == b"BGPO_OK"
     assert L.bgpo_status_string(8) == b"BGPO_ERR_TIMEOUT"
+    assert L.bgpo_status_string(9) == b"BGPO_ERR_BOUNDS"
     assert bg.kernel_name(2) == "lmhead_fwd_lse"
     assert bg.kernel_name(99) == "?"
 
@@ -207,3 +208,15 @@ def test_selftest_rejects_bad_arguments(L):
     assert L.bgpo_selftest_bounded_wait(FAKE + 8, 1024, 100, None) == 3
     assert L.bgpo_selftest_bounded_wait(FAKE, 1024, 0, None) == 1
     assert L.bgpo_selftest_bounded_wait(FAKE, 1024, 2000000, None) == 1
+
+
+def test_checked_build_exports_the_same_abi():
+    # the bounds-checked build (-DBGPO_CHECKED) is a drop-in for the normal one
+    from paper_2510_11683_gb300 import _lib
+    from tests.harness import ensure_built
+    h = ctypes.CDLL(ensure_built(checked=True))
+    for name, (res, args) in _lib.SIGNATURES.items():
+        f = getattr(h, name)
+        f.restype, f.argtypes = res, args
+    assert h.bgpo_abi_version() == 2
+    assert h.bgpo_status_string(9) == b"BGPO_ERR_BOUNDS"
