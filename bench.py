@@ -41,8 +41,8 @@ UNIT = "tokens/s"
 # masked rows M (the dW read-modify-write is fixed, dZ / Xm reads grow with M).
 # Valid only while the GEMM sources hash to `sha`.
 TRAFFIC = {
-    "dw_gemm": {"fixed_bytes": 4.0171e+09, "bytes_per_row": 353320.7,
-                "sha": "ef1569afb7fba77960e8ba13e1584f385ab49ab995479888074c54fcde49e576"},
+    "dw_gemm": {"fixed_bytes": 4.0064e+09, "bytes_per_row": 358778.3,
+                "sha": "7d2e48e77fce05458e7d23dadeb1f177edb847711c82ac5d51bc41e04da68271"},
 }
 
 
