@@ -436,3 +436,26 @@ def test_whole_step_replays_from_a_cuda_graph(bg, keep):
     assert bg.get_device_error(ws) == (0, 0)
     for k in ("ell", "coef", "dX", "dW"):
         assert torch.equal(graphed[k], eager[k]), k
+
+
+@pytest.mark.parametrize("shape", [
+    dict(B=1, P=0, R=1, H=64, V=1, n_t=1, G=1),      # one token, one-word vocabulary: l = 0
+    dict(B=2, P=0, R=5, H=64, V=2, n_t=1, G=2),      # no prompt, two-word vocabulary
+    dict(B=3, P=0, R=70, H=128, V=65, n_t=2, G=3),   # V one past a 64-column boundary
+])
+def test_degenerate_shapes_match_oracle(bg, shape):
+    import torch
+    wl = CONFIGS["tiny"].with_(name="degenerate", seed=77, **shape)
+    inp_cpu = make_inputs(wl)
+    inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
+    g = gpu_run(wl, inp)
+    o = oracle_run(wl, inp_cpu)
+    assert bg.get_device_error(g["ws"]) == (0, 0)
+    assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+    assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= ELL_TOL
+    # (with V = 1 the oracle's l and gradients are exactly zero; normwise then
+    # measures the absolute size of what the GPU returns)
+    assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL
+    assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL
+    if wl.V == 1:
+        assert float(g["ell"].abs().max()) <= 1e-4
