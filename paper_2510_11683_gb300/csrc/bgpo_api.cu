@@ -322,7 +322,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   const WsPtrs w = ws_pointers(ws, L);
 
   const bool keep = w.zc != nullptr;
-  CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xm_mn;
+  CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xmT_k;
   CUtensorMap map_dz_st, map_dxp_st, map_dw_red;
   const uint64_t dxp_rows = (uint64_t)dxp_row_block_cap(g) * kPairM;
   if (!map_2d(&map_xm_k, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
@@ -330,7 +330,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
       !map_2d(&map_dz_k, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, kBK, kBM) ||
       !map_2d(&map_w_mn, W, g.H, g.V, g.H * 2, 64, kBK) ||
       !map_2d(&map_dz_mn, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, kBK) ||
-      !map_2d(&map_xm_mn, w.xm, g.H, g.m_pad, g.H * 2, 64, kBK) ||
+      !map_2d(&map_xmT_k, w.xmT, g.m_pad, g.H, g.m_pad * 2, kBK, kBNHalf) ||
       // epilogue destinations: 32-row sub-tiles of 128 bytes
       !map_2d(&map_dz_st, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, 32) ||
       !map_2d(&map_dxp_st, w.dxp, g.H, dxp_rows, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32) ||
@@ -361,8 +361,12 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
     if (launch_dx_reduce(g, j, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
   {
+    TraceScope ts(prob->trace, KID_XM_TRANSPOSE, s);
+    if (launch_xm_transpose(g, j, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  {
     TraceScope ts(prob->trace, KID_DW_GEMM, s);
-    if (launch_gemm(GEMM_DW, map_dz_mn, map_xm_mn, map_dw_red, ga, w, s) != cudaSuccess)
+    if (launch_gemm(GEMM_DW, map_dz_mn, map_xmT_k, map_dw_red, ga, w, s) != cudaSuccess)
       return BGPO_ERR_CUDA;
   }
   return BGPO_OK;
@@ -472,7 +476,7 @@ const char* bgpo_kernel_name(int32_t id) {
   static const char* names[KID_COUNT] = {
       "mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
       "bound_coeffs", "lmhead_dz",   "dx_gemm",        "dx_reduce",   "dw_gemm",
-      "group_advantage", "selftest_wait", "vrpo_coeffs", "dz_from_logits"};
+      "group_advantage", "selftest_wait", "vrpo_coeffs", "dz_from_logits", "xm_transpose"};
   return (id >= 0 && id < KID_COUNT) ? names[id] : "?";
 }
 

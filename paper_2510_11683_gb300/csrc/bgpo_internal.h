@@ -22,6 +22,7 @@ struct WsPtrs {
   float* logp;
   float2* part;
   void* xm;   // bf16
+  void* xmT;  // bf16 [H, m_pad]
   void* dz;   // bf16
   float* dxp;
   float* zc;  // fp32 logits kept by the forward; null when the layout has none
@@ -54,6 +55,8 @@ cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const 
                                 float* g_out, const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* dX,
                              cudaStream_t s);
+// Xm^T from Xm for the current sample's rows (the dW GEMM reads it K-major).
+cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
                                    cudaStream_t s);
 cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,

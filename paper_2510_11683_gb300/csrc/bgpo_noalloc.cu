@@ -88,6 +88,7 @@ FwdLayout forward_layout(const Geometry& g) {
   L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
   L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
+  L.xmT = 0;       // forward only
   L.dz = 0;
   L.dxp = 0;
   L.dxp_elems = 0;

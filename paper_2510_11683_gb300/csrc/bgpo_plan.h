@@ -50,7 +50,8 @@ enum KernelId : int32_t {
   KID_SELFTEST_WAIT = 11,
   KID_VRPO_COEFFS = 12,
   KID_DZ_FROM_LOGITS = 13,
-  KID_COUNT = 14
+  KID_XM_TRANSPOSE = 14,
+  KID_COUNT = 15
 };
 
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -118,6 +119,7 @@ struct WsLayout {
   size_t logp;       // float[m_pad] log p(y_r)
   size_t part;       // float2[m_pad * n_vt] (max, sum-exp) per (row, vocab tile)
   size_t xm;         // bf16[m_pad * H] gathered masked hidden states
+  size_t xmT;        // bf16[H * m_pad] the same, transposed (the dW GEMM's K-major operand)
   size_t dz;         // bf16[m_pad * v_pad] dL/dz of the current sample
   size_t dxp;        // float[dxp_elems] split-K partials of dX
   size_t dxp_elems;
@@ -151,6 +153,7 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
   L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
   L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
+  L.xmT = o;       o = align_ws(o + 2 * (size_t)g.H * (size_t)g.m_pad);
   L.dz = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.v_pad);
   L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;
   L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
