@@ -41,8 +41,8 @@ UNIT = "tokens/s"
 # masked rows M (the dW read-modify-write is fixed, dZ / Xm reads grow with M).
 # Valid only while the GEMM sources hash to `sha`.
 TRAFFIC = {
-    "dw_gemm": {"fixed_bytes": 4.0064e+09, "bytes_per_row": 358778.3,
-                "sha": "7d2e48e77fce05458e7d23dadeb1f177edb847711c82ac5d51bc41e04da68271"},
+    "dw_gemm": {"fixed_bytes": 4.0215e+09, "bytes_per_row": 355490.8,
+                "sha": "c2e00d34dc0812313b44af7b9fa42b7615230ca6a2a1ec9c632c4fc03f569867"},
 }
 
 
