@@ -1,10 +1,9 @@
 """The bounds-checked build (-DBGPO_CHECKED) on the GPU.
 
-compute-sanitizer is not available on the GPU machines this library is tested
-on, so the library ships a build whose kernels test every index they read from
-device memory (masked-row lists, segment offsets, row counts) and every target
-token before use, recording BGPO_ERR_BOUNDS instead of touching memory out of
-bounds. Here the parity workloads run through that build, in a child process
+The library ships a build whose kernels test every index they read from device
+memory (masked-row lists, segment offsets, row counts) and every target token
+before use, recording BGPO_ERR_BOUNDS instead of touching memory out of bounds:
+a memory checker built into the library, usable where no external one runs. Here the parity workloads run through that build, in a child process
 that loads it (BGPO_LIBRARY=checked): the error word must stay clear and the
 results must match the oracle as the normal build's do, in both logit modes.
 A target token outside the vocabulary, which the normal build cannot see (it
