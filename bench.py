@@ -438,10 +438,15 @@ def main():
         del ws_keep
         torch.cuda.empty_cache()
 
-    if rank == 0 and world == 1 and not args.no_e2e:
-        out["e2e"] = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev, b_offset)
-    elif rank == 0 and world > 1:
-        out["e2e"] = None
+    if not args.no_e2e:
+        # every rank times its own shard end to end; whole job = all ranks'
+        # tokens over the slowest rank's time
+        e = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev, b_offset, barrier)
+        e_ms, e_tokens = aggregate_ranks(e["ms_per_step"], masked_per_step)
+        e.update(value=e_tokens / (e_ms / 1e3), ms_per_step=e_ms,
+                 h2d_bytes_per_step=e["h2d_bytes_per_step"] * world,
+                 d2h_bytes_per_step=e["d2h_bytes_per_step"] * world)
+        out["e2e"] = e
 
     if rank == 0 and world == 1 and not args.no_sweep:
         del dX, dW
@@ -460,7 +465,8 @@ def main():
         dist.destroy_process_group()
 
 
-def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0):
+def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0,
+            barrier=lambda: None):
     """Same step through host buffers: every step copies its inputs (X, W, Y,
     rewards or A, l_old) from pinned host memory and reads its results (l and g)
     back. Copies run on a second stream into the other of two device buffer
@@ -529,10 +535,12 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     run(max(1, min(args.warmup, 2)))
     torch.cuda.synchronize()
     steps = max(2, args.steps)   # the first step's copies are exposed once per run
+    barrier()
     t0 = time.perf_counter()
     run(steps)
     torch.cuda.synchronize()
     dt = (time.perf_counter() - t0) / steps
+    barrier()
     return {"value": masked_per_step / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps,
             "pipelining": "inputs of step k+1 copied on a second stream during step k"}
