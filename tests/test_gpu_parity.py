@@ -460,3 +460,23 @@ def test_degenerate_shapes_match_oracle(bg, shape):
     assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL
     if wl.V == 1:
         assert float(g["ell"].abs().max()) <= 1e-4
+
+
+def test_peak_device_memory_flat_in_n_t(bg):
+    # Linearity (Sec. 3): one sample's state at a time, so the device memory a
+    # step needs does not grow with n_t; only the caller's [n_t, B] vectors do
+    import torch
+    peaks = {}
+    for n_t in (1, 4, 16):
+        wl = CONFIGS["ragged"].with_(n_t=n_t)
+        inp = make_inputs(wl, device="cuda")     # same X, W, Y for every n_t (same seed)
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats()
+        base = torch.cuda.memory_allocated()
+        g = gpu_run(wl, inp)
+        assert bg.get_device_error(g["ws"]) == (0, 0)
+        peaks[n_t] = torch.cuda.max_memory_allocated() - base
+        del g, inp
+    vectors = 16 * 4 * wl.B * 8          # [n_t, B] float vectors of the harness, generously
+    assert peaks[16] - peaks[1] <= vectors + (1 << 20), peaks

@@ -93,3 +93,43 @@ def test_shard_of_assigns_disjoint_global_sequences():
     assert bench.shard_of(wl, 0, 1) == (wl, 0)
     seeds = {bench.shard_of(wl, r, 8)[0].seed for r in range(8)}
     assert len(seeds) == 8
+
+
+def _lost_rank_main(rank, port, out_dir):
+    # rank 1 leaves after its shard's work and before the dW sum; rank 0 must
+    # learn of it from the failed collective (or the group's short timeout)
+    # instead of hanging, and stop between steps with nothing in flight
+    import datetime
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=WORLD,
+                            timeout=datetime.timedelta(seconds=20))
+    wl = _workload()
+    inp = make_inputs(wl)
+    nb = wl.B // WORLD
+    b0 = rank * nb
+    X, W, Y = to64(inp["X"])[b0:b0 + nb], to64(inp["W"]), to64(inp["Y"])[b0:b0 + nb]
+    ts, masks = O.sample_masks(wl.seed, nb, wl.R, wl.n_t, wl.t_mode, b_offset=b0)
+    ell = O.elbo_all(X, W, Y, wl.P, ts, masks)
+    out = O.bgpo_step(X, W, Y, wl.P, oracle_advantages(wl, inp)[b0:b0 + nb], ell, ts, masks,
+                      1.0 / wl.G)
+    if rank == 1:
+        return                                     # leaves without joining the sum
+    dW = torch.from_numpy(out["dW"])
+    try:
+        dist.all_reduce(dW)
+        result = "completed"
+    except Exception as e:                         # noqa: BLE001 - any collective failure
+        result = "detected: " + type(e).__name__
+    with open(os.path.join(out_dir, "rank0.txt"), "w") as f:
+        f.write(result)
+
+
+def test_lost_rank_is_detected_by_the_survivor(tmp_path):
+    import time
+    t0 = time.time()
+    mp.spawn(_lost_rank_main, args=(_free_port(), str(tmp_path)), nprocs=WORLD, join=True)
+    with open(os.path.join(str(tmp_path), "rank0.txt")) as f:
+        result = f.read()
+    assert result.startswith("detected"), result
+    assert time.time() - t0 < 120
