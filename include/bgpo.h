@@ -317,7 +317,9 @@ bgpo_status bgpo_selftest_bounded_wait(void* ws, size_t ws_bytes, uint32_t timeo
 
 /* ---- per-kernel timing (host objects holding CUDA events) ---------------- */
 
-/* Creates a trace that can hold `capacity` kernel launches; NULL on failure. */
+/* Creates a trace that can hold `capacity` kernel launches; NULL on failure.
+ * A trace records from one host thread at a time: calls that may run
+ * concurrently need their own traces. */
 bgpo_trace* bgpo_trace_create(int32_t capacity);
 void bgpo_trace_destroy(bgpo_trace* trace);
 /* Forgets recorded launches (events are reused). */

@@ -374,13 +374,15 @@ def test_bounded_wait_times_out_and_context_survives(bg):
     assert torch.isfinite(ell).all()
 
 
-def test_variable_length_responses(bg):
+@pytest.mark.parametrize("keep", [False, True])
+def test_variable_length_responses(bg, keep):
     """Padded batches: positions at or past resp_len[b] are never masked and get
-    no gradient; everything else matches the oracle on the same draws."""
+    no gradient; everything else matches the oracle on the same draws (both
+    logit modes)."""
     wl = CONFIGS["ragged"]
     inp = make_inputs(wl, device="cuda")
     lens = np.array([301, 0, 117])
-    g = gpu_run(wl, inp, resp_len=lens)
+    g = gpu_run(wl, inp, resp_len=lens, keep_logits=keep)
     o = oracle_run(wl, {k: (v.cpu() if v is not None else None) for k, v in inp.items()},
                    resp_len=lens)
     assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
