@@ -74,8 +74,10 @@ CONFIGS = {
                         seed=5, targets="zipf", zipf_s=1.2, advantages="bernoulli",
                         eps_std=0.1),
     # parity cases spanning several tiles with ragged tails in every dimension
+    # (advantages drawn directly: one group of 3 Bernoulli rewards can be all
+    # equal, which makes every advantage, and every gradient, exactly zero)
     "ragged": Workload("ragged", B=3, P=5, R=301, H=192, V=1000, n_t=3, G=3, t_mode=0, seed=11,
-                       targets="zipf", zipf_s=1.1, advantages="bernoulli", eps_std=0.1),
+                       targets="zipf", zipf_s=1.1, advantages="normal", eps_std=0.1),
     "ragged_strat": Workload("ragged_strat", B=5, P=3, R=130, H=320, V=777, n_t=5, G=5,
                              t_mode=1, seed=12, targets="uniform", advantages="normal",
                              eps_std=0.3),
