@@ -14,8 +14,13 @@ host<->device copies inside the timed region; `roofline` = the dominant kernel's
 algorithmic tensor FLOP/s against the measured bf16 peak; `cpu_baseline` = the
 fp64 oracle on a bounded sample of the same workload on the host cores.
 `--impl reference` times that oracle alone (the reference arm of this tier).
-`keep_logits` = the same step with BGPO_FLAG_KEEP_LOGITS (the forward keeps its
-fp32 logits, the backward reads them instead of recomputing them).
+
+The step runs with BGPO_FLAG_PAIR_DW (MC samples 2k and 2k + 1 share one dW
+GEMM; the loop above is exactly the call order that flag expects) unless
+`--no-pair-dw` is given. `unpaired` = the same step without it (the library's
+default flags); `keep_logits` = the same step with BGPO_FLAG_KEEP_LOGITS too
+(the forward keeps its fp32 logits, the backward reads them instead of
+recomputing them).
 """
 import argparse
 import hashlib
@@ -35,14 +40,20 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of dw_gemm, from the
-# ncu capture of all 16 launches of the llada8b_r512_b8 case summarised in
-# profiles/dw_gemm_traffic_llada8b_r512_b8.md: an affine fit in the launch's
-# masked rows M (the dW read-modify-write is fixed, dZ / Xm reads grow with M).
-# Valid only while the GEMM sources hash to `sha`.
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind, from
+# the ncu capture of every GEMM launch of one llada8b_r512_b8 step (dW paired)
+# summarised in profiles/gemm_traffic_llada8b_r512_b8.md: affine fits in the
+# launch's rows (M, or K rows for dW). Valid only while the GEMM sources hash to
+# `sha`.
 TRAFFIC = {
-    "dw_gemm": {"fixed_bytes": 4.0215e+09, "bytes_per_row": 355490.8,
-                "sha": "c2e00d34dc0812313b44af7b9fa42b7615230ca6a2a1ec9c632c4fc03f569867"},
+    "lmhead_fwd_lse": {"fixed_bytes": 1.0261e+09, "bytes_per_row": 30290.0,
+           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
+    "lmhead_dz": {"fixed_bytes": 9.8207e+08, "bytes_per_row": 356492.7,
+           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
+    "dx_gemm": {"fixed_bytes": 6.1442e+08, "bytes_per_row": 1290212.4,
+           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
+    "dw_gemm": {"fixed_bytes": 2.2937e+09, "bytes_per_row": 1220896.5,
+           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
 }
 
 
@@ -57,7 +68,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-keep-logits", action="store_true",
-                    help="skip the second timed leg with BGPO_FLAG_KEEP_LOGITS")
+                    help="skip the timed leg with BGPO_FLAG_KEEP_LOGITS")
+    ap.add_argument("--no-pair-dw", action="store_true",
+                    help="time the step without BGPO_FLAG_PAIR_DW (and skip the unpaired leg)")
     ap.add_argument("--grad-variance", action="store_true",
                     help="run the Sec. 4.3 gradient std / bias vs n_t study instead")
     return ap.parse_args()
@@ -280,7 +293,8 @@ def main():
     X, W, Y = inp["X"], inp["W"], inp["Y"]
     n_t, Bsz = wl.n_t, wl.B
 
-    prob = bg.problem_from(wl, b_offset=b_offset)
+    pair = not args.no_pair_dw
+    prob = bg.problem_from(wl, b_offset=b_offset, pair_dw=pair)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     A = torch.empty(Bsz, dtype=torch.float32, device=dev)
@@ -311,7 +325,7 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
-    def timed_leg(keep, ws_, sample_clocks):
+    def timed_leg(keep, pair_dw, ws_, sample_clocks):
         """W warm-up and K timed steps of one mode; per-kernel times from the trace."""
         def step(p):
             for j in range(n_t):
@@ -321,10 +335,11 @@ def main():
                 bg.elbo_bwd_accumulate(p, j, X, W, Y, coef[j], ws_, dX, dW)
 
         for _ in range(args.warmup):
-            step(bg.problem_from(wl, b_offset=b_offset, keep_logits=keep))
+            step(bg.problem_from(wl, b_offset=b_offset, keep_logits=keep, pair_dw=pair_dw))
         torch.cuda.synchronize()
         trace = bg.Trace(args.steps * n_t * 12 + 16)
-        prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset, keep_logits=keep)
+        prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset, keep_logits=keep,
+                                 pair_dw=pair_dw)
         clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
         stream = torch.cuda.current_stream()
         e0 = torch.cuda.Event(enable_timing=True)
@@ -368,7 +383,9 @@ def main():
         achieved = dom_flops_per_launch / dom_avg_s / 1e12
         traffic = None
         if dom in TRAFFIC and TRAFFIC[dom]["sha"] == kernel_sha():
-            traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * masked_per_step / n_t
+            # K rows of an average launch (two samples' rows when dW pairs them)
+            rows_per_launch = masked_per_step * args.steps / dom_launches
+            traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * rows_per_launch
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
@@ -385,8 +402,8 @@ def main():
                         "peak_kind": f"HBM copy ({peaks['source']})"}
         return roof, hbm_pass, len(gemm_kernels)
 
-    # headline: the default mode (logits recomputed in the backward, never stored)
-    ms_local, per_kernel, clock_info, gpu_launches = timed_leg(False, ws, True)
+    # headline: logits recomputed in the backward, never stored; dW paired
+    ms_local, per_kernel, clock_info, gpu_launches = timed_leg(False, pair, ws, True)
     ms, masked_all = aggregate_ranks(ms_local, masked_per_step)
     roofline, _, n_gemm = rooflines(per_kernel)
     value = masked_all / (ms / 1e3)
@@ -399,6 +416,7 @@ def main():
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; shapes of the paper's "
         "LLaDA-8B head, response 512, n_t=16)", "config": config_of(wl),
         "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clock_info,
+        "library_flags": ["BGPO_FLAG_PAIR_DW"] if pair else [],
         "mc_samples_per_s": Bsz * n_t * world / (ms / 1e3),
         "masked_rows_per_step": masked_per_step, "masked_rows_per_sample": rows_per_sample,
         "step_tensor_tflops_executed": exec_tflops,
@@ -414,14 +432,28 @@ def main():
               f"{ {k: round(v[1] / args.steps, 3) for k, v in per_kernel.items()} }",
               file=sys.stderr, flush=True)
 
+    # the same step with the library's default flags (a dW GEMM per sample)
+    if rank == 0 and world == 1 and pair:
+        u_ms, u_per_kernel, _, u_launches = timed_leg(False, False, ws, False)
+        u_roof, _, _ = rooflines(u_per_kernel)
+        out["unpaired"] = {
+            "value": masked_per_step / (u_ms / 1e3), "unit": UNIT, "ms_per_step": u_ms,
+            "gpu_launches": u_launches, "roofline": u_roof,
+            "per_kernel_ms_per_step": {k: v[1] / args.steps for k, v in u_per_kernel.items()}}
+        print(f"[bench] unpaired: {u_ms:.2f} ms/step, {masked_per_step / (u_ms / 1e3):.4g} tok/s, "
+              f"per kernel ms/step: "
+              f"{ {k: round(v[1] / args.steps, 3) for k, v in u_per_kernel.items()} }",
+              file=sys.stderr, flush=True)
+
     # the same step with BGPO_FLAG_KEEP_LOGITS (the forward keeps its fp32 logits,
     # the backward forms dL/dz from them in one HBM pass instead of a fourth GEMM)
     if rank == 0 and world == 1 and not args.no_keep_logits:
         del ws
         torch.cuda.empty_cache()
         torch.cuda.reset_peak_memory_stats(dev)
-        ws_keep = bg.alloc_workspace(bg.problem_from(wl, b_offset=b_offset, keep_logits=True), dev)
-        k_ms, k_per_kernel, _, k_launches = timed_leg(True, ws_keep, False)
+        ws_keep = bg.alloc_workspace(
+            bg.problem_from(wl, b_offset=b_offset, keep_logits=True, pair_dw=pair), dev)
+        k_ms, k_per_kernel, _, k_launches = timed_leg(True, pair, ws_keep, False)
         k_roof, k_hbm, _ = rooflines(k_per_kernel)
         out["keep_logits"] = {
             "value": masked_per_step / (k_ms / 1e3), "unit": UNIT, "ms_per_step": k_ms,
@@ -441,7 +473,8 @@ def main():
     if not args.no_e2e:
         # every rank times its own shard end to end; whole job = all ranks'
         # tokens over the slowest rank's time
-        e = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev, b_offset, barrier)
+        e = e2e_leg(bg, wl, inp_cpu, ell_old.cpu(), masked_per_step, args, dev, b_offset, barrier,
+                    pair)
         e_ms, e_tokens = aggregate_ranks(e["ms_per_step"], masked_per_step)
         e.update(value=e_tokens / (e_ms / 1e3), ms_per_step=e_ms,
                  h2d_bytes_per_step=e["h2d_bytes_per_step"] * world,
@@ -451,7 +484,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_sweep:
         del dX, dW
         torch.cuda.empty_cache()
-        out["nt_sweep"] = nt_sweep(bg, dev)
+        out["nt_sweep"] = nt_sweep(bg, dev, pair)
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rows, dt, desc = oracle_sample(wl, inp_cpu)
@@ -466,7 +499,7 @@ def main():
 
 
 def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0,
-            barrier=lambda: None):
+            barrier=lambda: None, pair=False):
     """Same step through host buffers: every step copies its inputs (X, W, Y,
     rewards or A, l_old) from pinned host memory and reads its results (l and g)
     back. Copies run on a second stream into the other of two device buffer
@@ -483,7 +516,7 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     bufs = [{k: torch.empty_like(v, device=dev) for k, v in host.items()} for _ in range(2)]
     out_ell = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
     out_g = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
-    prob = bg.problem_from(wl, b_offset=b_offset)
+    prob = bg.problem_from(wl, b_offset=b_offset, pair_dw=pair)
     ws = bg.alloc_workspace(prob, dev)
     A = torch.empty(Bsz, dtype=torch.float32, device=dev)
     ell = torch.empty((n_t, Bsz), dtype=torch.float32, device=dev)
@@ -623,12 +656,14 @@ def run_grad_variance(args, wl):
 CONFIG_GRAD_VARIANCE = {"n_t": (1, 2, 4, 8, 16, 32), "repeats": 8, "golden_n_t": 256}
 
 
-def nt_sweep(bg, dev):
+def nt_sweep(bg, dev, pair=False):
     """Time and peak memory of one step vs n_t (8 x (256 + 512), LLaDA-8B head) for
     BGPO and for the ELBO-based objective it bounds (VRPO, Eq. 7), whose weights
     need every sample's l first: "vrpo_retain" keeps one workspace per sample
     (memory grows with n_t), "vrpo_recompute" runs each sample's forward twice.
-    Every backward recomputes its logits (the default mode)."""
+    Every backward recomputes its logits. `pair`: BGPO and vrpo_recompute pair
+    the dW GEMMs of samples 2k and 2k + 1 (vrpo_retain, one workspace per
+    sample, cannot)."""
     import torch
     from synth import CONFIGS, SWEEP_NT, make_inputs
     base = CONFIGS["llada8b_sweep"]
@@ -654,7 +689,8 @@ def nt_sweep(bg, dev):
             torch.cuda.empty_cache()
             torch.cuda.reset_peak_memory_stats(dev)
             n_ws = n_t if method == "vrpo_retain" else 1
-            wss = [bg.alloc_workspace(prob, dev) for _ in range(n_ws)]
+            pm = bg.problem_from(wl, pair_dw=pair and method != "vrpo_retain")
+            wss = [bg.alloc_workspace(pm, dev) for _ in range(n_ws)]
             ell = torch.empty((n_t, wl.B), dtype=torch.float32, device=dev)
             coef, g = torch.empty_like(ell), torch.empty_like(ell)
             cv = torch.empty(wl.B, dtype=torch.float32, device=dev)
@@ -666,22 +702,22 @@ def nt_sweep(bg, dev):
                 if method == "bgpo":
                     ws = wss[0]
                     for j in range(n_t):
-                        bg.sample_mask(prob, j, ws)
-                        bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
-                        bg.bound_coeffs(prob, j, ell[j], ell[j], A, coef[j], g[j], ws)
-                        bg.elbo_bwd_accumulate(prob, j, X, W, Y, coef[j], ws, dX, dW)
+                        bg.sample_mask(pm, j, ws)
+                        bg.elbo_fwd(pm, j, X, W, Y, ws, ell[j])
+                        bg.bound_coeffs(pm, j, ell[j], ell[j], A, coef[j], g[j], ws)
+                        bg.elbo_bwd_accumulate(pm, j, X, W, Y, coef[j], ws, dX, dW)
                     return
                 for j in range(n_t):
                     ws = wss[j % n_ws]
-                    bg.sample_mask(prob, j, ws)
-                    bg.elbo_fwd(prob, j, X, W, Y, ws, ell[j])
-                bg.vrpo_coeffs(prob, ell, ell, A, cv, None, wss[0])
+                    bg.sample_mask(pm, j, ws)
+                    bg.elbo_fwd(pm, j, X, W, Y, ws, ell[j])
+                bg.vrpo_coeffs(pm, ell, ell, A, cv, None, wss[0])
                 for j in range(n_t):
                     ws = wss[j % n_ws]
                     if method == "vrpo_recompute":
-                        bg.sample_mask(prob, j, ws)
-                        bg.elbo_fwd(prob, j, X, W, Y, ws, tmp)
-                    bg.elbo_bwd_accumulate(prob, j, X, W, Y, cv, ws, dX, dW)
+                        bg.sample_mask(pm, j, ws)
+                        bg.elbo_fwd(pm, j, X, W, Y, ws, tmp)
+                    bg.elbo_bwd_accumulate(pm, j, X, W, Y, cv, ws, dX, dW)
             run()
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -690,8 +726,12 @@ def nt_sweep(bg, dev):
             e1.record()
             torch.cuda.synchronize()
             ms = e0.elapsed_time(e1)
+            code = bg.get_device_error(wss[0])[0]
+            if code != 0:
+                raise RuntimeError(f"n_t sweep {method}: device error {code}")
             point[method] = {"ms": ms, "tokens_per_s": rows / (ms / 1e3),
-                             "peak_bytes": torch.cuda.max_memory_allocated(dev)}
+                             "peak_bytes": torch.cuda.max_memory_allocated(dev),
+                             "dw_paired": bool(pm.flags & bg.FLAG_PAIR_DW)}
             del wss, dX, dW
         res.append(point)
     return res

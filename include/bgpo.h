@@ -100,6 +100,29 @@ typedef struct bgpo_trace bgpo_trace;
  *       for forward-only passes (the old policy's l_old).
  */
 #define BGPO_FLAG_KEEP_LOGITS 1u
+/*
+ *   BGPO_FLAG_PAIR_DW  consecutive MC samples (2k, 2k + 1) share one dW GEMM
+ *       whose K range holds both samples' masked rows (M_2k + M_2k+1 instead
+ *       of M_j), so dW's fp32 read-modify-write (8 V H bytes) happens once per
+ *       pair instead of once per sample. The backward of an even sample j < n_t - 1
+ *       updates dX as usual but leaves its dL/dz rows and gathered hidden
+ *       states pending in the workspace and adds nothing to dW; the backward of
+ *       sample j + 1 on the same workspace adds both samples' dW contributions.
+ *       dW is therefore complete after the backward of every odd sample and of
+ *       the last sample (j = n_t - 1), i.e. at the end of Algorithm 1's loop,
+ *       but not between the two backward calls of a pair. The same dW up to
+ *       fp32 summation order; dX and l are unchanged bit for bit. The dZ and
+ *       Xm^T regions of the workspace double: 2 * roundup(B R, 256) *
+ *       (roundup(V, 64) + H) more bytes, independent of n_t. Every call on
+ *       the workspace within a step must carry the flag. Misuse is reported in
+ *       the device error word as BGPO_ERR_INVALID_ARG: the backward of an odd
+ *       sample whose partner is not pending (its dW then holds sample j
+ *       alone), or the masking of another sample while one is pending (the
+ *       pending contribution is dropped). bgpo_clear_device_error forgets a
+ *       pending sample. Keeping every sample's workspace apart (bgpo_vrpo_coeffs'
+ *       "retain" strategy) does not pair: leave the flag off there.
+ */
+#define BGPO_FLAG_PAIR_DW 2u
 
 /*
  * Problem description (host struct, read by every call; never stored).
@@ -159,10 +182,9 @@ bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
 
 /*
  * Bytes of device workspace the calls below need for `prob`. Depends on B, R,
- * H, V and BGPO_FLAG_KEEP_LOGITS only -- never on n_t (Linearity, Sec. 3:
- * one sample's state at a time). The layout without the logits is a prefix of
- * the layout with them, so a workspace sized with the flag also serves calls
- * made without it. Returns 0 for an invalid problem.
+ * H, V and the flags only -- never on n_t (Linearity, Sec. 3: one sample's
+ * state at a time; with BGPO_FLAG_PAIR_DW two). A workspace sized with a flag
+ * also serves calls made without it. Returns 0 for an invalid problem.
  */
 size_t bgpo_workspace_bytes(const bgpo_problem* prob);
 
@@ -244,6 +266,8 @@ bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const f
  *           on the tensor cores, or with BGPO_FLAG_KEEP_LOGITS read from what
  *           bgpo_elbo_fwd kept; the two give identical bits)
  *   dX[b, i, :] += W^T dz_r        dW += sum_r dz_r x_r^T
+ * (with BGPO_FLAG_PAIR_DW the dW term of an even sample is added by the next
+ * sample's call.)
  * coef is an input (normally bgpo_bound_coeffs' output for the same j).
  *   dX device float [B, R, H], dW device float [V, H]: accumulated in place.
  * Deterministic: no atomics, fixed summation order.
@@ -302,7 +326,9 @@ bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j, const voi
 bgpo_status bgpo_get_device_error(const void* ws, size_t ws_bytes, int32_t* code_out,
                                   int32_t* where_out, void* stream);
 
-/* Clears the device error word (asynchronous on `stream`). */
+/* Clears the device error word (asynchronous on `stream`) and forgets a
+ * sample pending under BGPO_FLAG_PAIR_DW. Clear a new workspace before its
+ * first call. */
 bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream);
 
 /*

@@ -19,6 +19,7 @@ from ._lib import BgpoError, BgpoProblem  # noqa: F401
 T_IID = 0
 T_STRATIFIED = 1
 FLAG_KEEP_LOGITS = 1   # BGPO_FLAG_KEEP_LOGITS
+FLAG_PAIR_DW = 2       # BGPO_FLAG_PAIR_DW
 
 
 def _torch():
@@ -27,7 +28,7 @@ def _torch():
 
 
 def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None,
-            b_offset=0, resp_len=None, keep_logits=False):
+            b_offset=0, resp_len=None, keep_logits=False, pair_dw=False):
     """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1).
 
     b_offset: global index of the first sequence (a data-parallel shard of a
@@ -36,7 +37,10 @@ def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=
     positions are never masked); the tensor must outlive the calls.
     keep_logits: sets BGPO_FLAG_KEEP_LOGITS (the forward keeps the masked
     rows' fp32 logits in the workspace and the backward reads them instead of
-    recomputing them; larger workspace, same results)."""
+    recomputing them; larger workspace, same results).
+    pair_dw: sets BGPO_FLAG_PAIR_DW (samples 2k and 2k + 1 share one dW GEMM:
+    dW is complete after every odd sample's backward and the last sample's,
+    not in between; larger workspace, dW equal up to fp32 summation order)."""
     p = BgpoProblem()
     p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
     p.seed = seed
@@ -44,17 +48,17 @@ def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=
     p.b_offset = b_offset
     p.resp_len = _ptr(resp_len, _torch().int32, "resp_len") if resp_len is not None else None
     p.trace = trace.handle if isinstance(trace, Trace) else trace
-    p.flags = FLAG_KEEP_LOGITS if keep_logits else 0
+    p.flags = (FLAG_KEEP_LOGITS if keep_logits else 0) | (FLAG_PAIR_DW if pair_dw else 0)
     p.reserved = 0
     return p
 
 
 def problem_from(wl, trace=None, loss_scale=None, b_offset=0, resp_len=None,
-                 keep_logits=False):
+                 keep_logits=False, pair_dw=False):
     """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
     return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
                    loss_scale=loss_scale, trace=trace, b_offset=b_offset, resp_len=resp_len,
-                   keep_logits=keep_logits)
+                   keep_logits=keep_logits, pair_dw=pair_dw)
 
 
 def validate_problem(prob):
@@ -70,7 +74,8 @@ def workspace_bytes(prob):
 
 def alloc_workspace(prob, device="cuda"):
     """A uint8 device tensor of workspace_bytes(prob) (256-byte aligned by torch)
-    with a cleared device error word (the rest is scratch the calls overwrite)."""
+    with a cleared device error word and nothing pending (the rest is scratch
+    the calls overwrite)."""
     torch = _torch()
     ws = torch.empty(workspace_bytes(prob), dtype=torch.uint8, device=device)
     assert ws.data_ptr() % 256 == 0

@@ -65,7 +65,8 @@ bgpo_status check_problem(const bgpo_problem* p) {
   if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
   if (p->b_offset < 0) return BGPO_ERR_INVALID_ARG;
   if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
-  if ((p->flags & ~BGPO_FLAG_KEEP_LOGITS) != 0u || p->reserved != 0) return BGPO_ERR_INVALID_ARG;
+  if ((p->flags & ~(BGPO_FLAG_KEEP_LOGITS | BGPO_FLAG_PAIR_DW)) != 0u || p->reserved != 0)
+    return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
   if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
@@ -79,6 +80,8 @@ Geometry geometry_of(const bgpo_problem* p) { return make_geometry(p->B, p->P, p
 
 bool keeps_logits(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_KEEP_LOGITS) != 0u; }
 
+bool pairs_dw(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_PAIR_DW) != 0u; }
+
 bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
   return (j >= 0 && j < p->n_t) ? BGPO_OK : BGPO_ERR_INVALID_ARG;
 }
@@ -86,7 +89,7 @@ bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
 bgpo_status check_ws(const bgpo_problem* p, const void* ws, size_t ws_bytes, WsLayout* L) {
   if (!ws) return BGPO_ERR_INVALID_ARG;
   if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
-  *L = make_ws_layout(geometry_of(p), keeps_logits(p));
+  *L = make_ws_layout(geometry_of(p), keeps_logits(p), pairs_dw(p));
   if (ws_bytes < L->total) return BGPO_ERR_WORKSPACE_TOO_SMALL;
   return BGPO_OK;
 }
@@ -175,7 +178,7 @@ bgpo_status bgpo_validate_problem(const bgpo_problem* prob) { return check_probl
 
 size_t bgpo_workspace_bytes(const bgpo_problem* prob) {
   if (check_problem(prob) != BGPO_OK) return 0;
-  return make_ws_layout(geometry_of(prob), keeps_logits(prob)).total;
+  return make_ws_layout(geometry_of(prob), keeps_logits(prob), pairs_dw(prob)).total;
 }
 
 bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size_t ws_bytes,
@@ -203,6 +206,7 @@ bgpo_status bgpo_sample_mask(const bgpo_problem* prob, int32_t j, void* ws, size
   a.t_out = t_out;
   a.mask_out = mask_out;
   a.resp_len = prob->resp_len;
+  a.pair_dw = pairs_dw(prob);
   TraceScope ts(prob->trace, KID_MASK_COMPACT, s);
   return from_cuda(launch_mask_compact(a, w, s));
 }
@@ -322,17 +326,22 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   const WsPtrs w = ws_pointers(ws, L);
 
   const bool keep = w.zc != nullptr;
+  // dW pairing: an even sample's dW GEMM waits for the next sample's (unless it
+  // is the last sample); an odd sample's dW GEMM covers both samples' rows
+  const bool pair = pairs_dw(prob);
+  const bool defer = pair && j % 2 == 0 && j + 1 < prob->n_t;
+  const uint64_t zr = (uint64_t)w.dz_rows;
   CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xmT_k;
   CUtensorMap map_dz_st, map_dxp_st, map_dw_red;
   const uint64_t dxp_rows = (uint64_t)dxp_row_block_cap(g) * kPairM;
   if (!map_2d(&map_xm_k, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
       !map_2d(&map_w_k, W, g.H, g.V, g.H * 2, kBK, kBNHalf) ||
-      !map_2d(&map_dz_k, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, kBK, kBM) ||
+      !map_2d(&map_dz_k, w.dz, g.v_pad, zr, g.v_pad * 2, kBK, kBM) ||
       !map_2d(&map_w_mn, W, g.H, g.V, g.H * 2, 64, kBK) ||
-      !map_2d(&map_dz_mn, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, kBK) ||
-      !map_2d(&map_xmT_k, w.xmT, g.m_pad, g.H, g.m_pad * 2, kBK, kBNHalf) ||
+      !map_2d(&map_dz_mn, w.dz, g.v_pad, zr, g.v_pad * 2, 64, kBK) ||
+      !map_2d(&map_xmT_k, w.xmT, zr, g.H, zr * 2, kBK, kBNHalf) ||
       // epilogue destinations: 32-row sub-tiles of 128 bytes
-      !map_2d(&map_dz_st, w.dz, g.v_pad, g.m_pad, g.v_pad * 2, 64, 32) ||
+      !map_2d(&map_dz_st, w.dz, g.v_pad, zr, g.v_pad * 2, 64, 32) ||
       !map_2d(&map_dxp_st, w.dxp, g.H, dxp_rows, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32) ||
       !map_2d(&map_dw_red, dW, g.H, g.V, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32))
     return BGPO_ERR_CUDA;
@@ -343,6 +352,7 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   ga.coef = coef;
   ga.dW = dW;
   ga.dX = dX;
+  ga.pair_consume = pair && (j & 1);
   if (keep) {
     TraceScope ts(prob->trace, KID_DZ_FROM_LOGITS, s);
     if (launch_dz_from_logits(g, j, coef, sms, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
@@ -362,9 +372,9 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   }
   {
     TraceScope ts(prob->trace, KID_XM_TRANSPOSE, s);
-    if (launch_xm_transpose(g, j, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    if (launch_xm_transpose(g, j, defer, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
-  {
+  if (!defer) {
     TraceScope ts(prob->trace, KID_DW_GEMM, s);
     if (launch_gemm(GEMM_DW, map_dz_mn, map_xmT_k, map_dw_red, ga, w, s) != cudaSuccess)
       return BGPO_ERR_CUDA;
@@ -408,7 +418,16 @@ bgpo_status bgpo_clear_device_error(void* ws, size_t ws_bytes, void* stream) {
   if (!ws) return BGPO_ERR_INVALID_ARG;
   if (!aligned(ws, 256)) return BGPO_ERR_ALIGNMENT;
   if (ws_bytes < 64) return BGPO_ERR_WORKSPACE_TOO_SMALL;
-  return from_cuda(cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), static_cast<cudaStream_t>(stream)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // status and where to 0; the dW pairing state (ERR_PEND .. ERR_PAIRED) to -1:
+  // nothing pending
+  if (cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), s) != cudaSuccess ||
+      cudaMemsetAsync(static_cast<int32_t*>(ws) + ERR_PEND, 0xff, 4 * sizeof(int32_t), s) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return BGPO_ERR_CUDA;
+  }
+  return BGPO_OK;
 }
 
 bgpo_status bgpo_selftest_bounded_wait(void* ws, size_t ws_bytes, uint32_t timeout_us,

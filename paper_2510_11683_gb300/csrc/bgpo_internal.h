@@ -22,8 +22,9 @@ struct WsPtrs {
   float* logp;
   float2* part;
   void* xm;   // bf16
-  void* xmT;  // bf16 [H, m_pad]
-  void* dz;   // bf16
+  void* xmT;  // bf16 [H, dz_rows]
+  void* dz;   // bf16 [dz_rows, v_pad]
+  int64_t dz_rows;
   float* dxp;
   float* zc;  // fp32 logits kept by the forward; null when the layout has none
 };
@@ -37,6 +38,7 @@ struct MaskArgs {
   float* t_out;       // may be null
   uint8_t* mask_out;  // may be null
   const int32_t* resp_len;  // may be null: [B] real response lengths
+  bool pair_dw = false;     // BGPO_FLAG_PAIR_DW: an odd sample may pair with a pending one
 };
 
 cudaError_t launch_mask_compact(const MaskArgs& a, const WsPtrs& w, cudaStream_t s);
@@ -55,8 +57,11 @@ cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const 
                                 float* g_out, const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* dX,
                              cudaStream_t s);
-// Xm^T from Xm for the current sample's rows (the dW GEMM reads it K-major).
-cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s);
+// Xm^T from Xm for the current sample's rows (the dW GEMM reads it K-major),
+// from column ERR_ROW_OFF on. `defer`: this sample's dW GEMM waits for the
+// next sample's; the kernel records the sample as pending.
+cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, bool defer, const WsPtrs& w,
+                                cudaStream_t s);
 cudaError_t launch_group_advantage(int32_t B, int32_t G, const float* rewards, float* A_out,
                                    cudaStream_t s);
 cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
@@ -74,6 +79,7 @@ struct GemmArgs {
   const float* coef;  // GEMM_DZ: per-sequence dL/dl
   float* dW;          // GEMM_DW: accumulated weight gradient [V, H]
   float* dX = nullptr;  // GEMM_DX: accumulated dHidden [B, R, H] (written directly without split-K)
+  bool pair_consume = false;  // GEMM_DW: this dW GEMM completes a pair (odd j, BGPO_FLAG_PAIR_DW)
 };
 
 // CTA pairs the GEMM kernels run as: the 2-CTA clusters that fit on the

@@ -90,6 +90,7 @@ FwdLayout forward_layout(const Geometry& g) {
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
   L.xmT = 0;       // forward only
   L.dz = 0;
+  L.dz_rows = (size_t)g.m_pad;
   L.dxp = 0;
   L.dxp_elems = 0;
   L.zc = 0;        // keeps no logits

@@ -107,8 +107,7 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
 // Device workspace layout. Every region starts on a 1024-byte boundary (TMA
 // tiles with 128-byte swizzle want 1024-byte aligned bases).
 struct WsLayout {
-  size_t err;        // int32[16]: [0] status, [1] where, [2] sample tag j, [3] M, [4] logits kept,
-                     //            [5] dX split count
+  size_t err;        // int32[16]: the fields of ErrField
   size_t t;          // float[B]    t_{b,j}
   size_t tnum;       // uint32[2B]  T numerator (t = T / D), (low, high) words
   size_t seg_off;    // int32[B+1]  first compacted row of each sequence
@@ -119,8 +118,9 @@ struct WsLayout {
   size_t logp;       // float[m_pad] log p(y_r)
   size_t part;       // float2[m_pad * n_vt] (max, sum-exp) per (row, vocab tile)
   size_t xm;         // bf16[m_pad * H] gathered masked hidden states
-  size_t xmT;        // bf16[H * m_pad] the same, transposed (the dW GEMM's K-major operand)
-  size_t dz;         // bf16[m_pad * v_pad] dL/dz of the current sample
+  size_t xmT;        // bf16[H * dz_rows] the same, transposed (the dW GEMM's K-major operand)
+  size_t dz;         // bf16[dz_rows * v_pad] dL/dz of the current sample (and of a pending one)
+  size_t dz_rows;    // m_pad, or 2 m_pad when the dW GEMM pairs samples
   size_t dxp;        // float[dxp_elems] split-K partials of dX
   size_t dxp_elems;
   size_t zc;         // float[m_pad * v_pad] logits kept by the forward (last region)
@@ -137,11 +137,13 @@ BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
   return mb_max > kMaxSplits ? mb_max : kMaxSplits;
 }
 
-// `keep_logits` appends the fp32 logit region; every other region has the same
-// offset either way.
-BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
+// `keep_logits` appends the fp32 logit region. `pair_dw` doubles the rows of
+// dZ and the columns of Xm^T: the rows of an even sample wait there for the
+// dW GEMM of the next sample, whose rows follow them.
+BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits, bool pair_dw) {
   WsLayout L;
   size_t o = 0;
+  L.dz_rows = (pair_dw ? 2 : 1) * (size_t)g.m_pad;
   L.err = o;       o = align_ws(o + 64);
   L.t = o;         o = align_ws(o + 4 * (size_t)g.B);
   L.tnum = o;      o = align_ws(o + 8 * (size_t)g.B);
@@ -153,8 +155,8 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
   L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
   L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
-  L.xmT = o;       o = align_ws(o + 2 * (size_t)g.H * (size_t)g.m_pad);
-  L.dz = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.v_pad);
+  L.xmT = o;       o = align_ws(o + 2 * (size_t)g.H * L.dz_rows);
+  L.dz = o;        o = align_ws(o + 2 * L.dz_rows * (size_t)g.v_pad);
   L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;
   L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
   L.zc_bytes = keep_logits ? 4 * (size_t)g.m_pad * (size_t)g.v_pad : 0;
@@ -164,12 +166,37 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits) {
   return L;
 }
 
-// Indices into the int32 error word. ERR_LOGITS is 1 while the logit region
-// holds the current sample's logits (set by the forward that wrote them,
-// cleared by the masking of a new sample and by a forward that keeps none).
-// ERR_DX_SPLITS is the split-K count the last dX GEMM used.
+// Indices into the int32 error word:
+//   ERR_STATUS, ERR_WHERE  the device error (bgpo_get_device_error)
+//   ERR_SAMPLE, ERR_M      the sample j the workspace holds and its masked rows
+//   ERR_LOGITS    1 while the logit region holds the current sample's logits
+//                 (set by the forward that wrote them, cleared by the masking of
+//                 a new sample and by a forward that keeps none)
+//   ERR_DX_SPLITS the split-K count the last dX GEMM used
+//   ERR_PEND      pend_tag(j) while sample j's dZ and Xm^T rows wait for the dW
+//                 GEMM of sample j + 1, else -1
+//   ERR_PEND_OFF  the row at which sample j + 1's dZ and Xm^T rows start: M_j
+//                 rounded up to a K block
+//   ERR_ROW_OFF   set by the masking: the first dZ / Xm^T row of the current
+//                 sample (ERR_PEND_OFF when it pairs with the pending sample,
+//                 else 0)
+//   ERR_PAIRED    set by the masking: 1 when the current sample pairs
 enum ErrField : int {
-  ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4, ERR_DX_SPLITS = 5
+  ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4, ERR_DX_SPLITS = 5,
+  ERR_PEND = 6, ERR_PEND_OFF = 7, ERR_ROW_OFF = 8, ERR_PAIRED = 9
 };
+
+// Tag of a pending sample (n_t < 2^16): neither -1 nor a small integer that
+// memory not yet written by this library is likely to hold.
+BGPO_HD int32_t pend_tag(int32_t j) { return (int32_t)(0x5EED0000u | (uint32_t)j); }
+
+// First dZ / Xm^T row of the current sample, clamped to the room the layout
+// has for a pending sample (none without pairing) and to a K block.
+BGPO_HD int64_t row_offset(int32_t stored, int64_t dz_rows, int64_t m_pad) {
+  const int64_t room = dz_rows - m_pad;
+  int64_t off = stored < 0 ? 0 : (int64_t)stored;
+  if (off > room) off = room;
+  return off & ~(int64_t)(kBK - 1);
+}
 
 }  // namespace bgpo

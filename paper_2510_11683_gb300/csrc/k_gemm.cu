@@ -27,7 +27,8 @@
 //   GEMM_DX   dXm = dZ W (K = vocabulary): split-K partials in fp32, or, when
 //             the launch needs no split, added straight into the dX rows.
 //   GEMM_DW   dW += dZ^T Xm (K = masked rows; Xm read as its transpose, so
-//             that the B operand is K-major), fp32 TMA reduce-add.
+//             that the B operand is K-major), fp32 TMA reduce-add. With dW
+//             pairing, K also covers the rows of the pending sample before.
 //
 // Every wait is bounded (time and polls); a wait that runs out sets the
 // workspace error word to BGPO_ERR_TIMEOUT and both CTAs drain and exit.
@@ -58,6 +59,7 @@ struct GemmParams {
   const float* coef;
   float* dW;
   float* dX;
+  bool pair_consume;
 };
 
 struct Work {
@@ -69,8 +71,10 @@ struct Unit {
   int32_t m_blk, n_blk, split, kb0, kb_n;
 };
 
+// `roff`: the first dZ / Xm^T row of the sample (dW pairing; 0 otherwise). The
+// dW GEMM's K range [0, roff + M) then covers a pending sample's rows too.
 template <int KIND>
-__device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M) {
+__device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_t roff) {
   Work w;
   w.splits = 1;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
@@ -89,8 +93,8 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M) {
   } else {  // GEMM_DW
     w.tiles_m = ceil_div(p.g.V, kPairM);
     w.tiles_n = p.g.tiles_h;
-    w.kb_total = ceil_div(M, kBK);
-    w.units = M > 0 ? w.tiles_m * w.tiles_n : 0;
+    w.kb_total = ceil_div(roff + M, kBK);
+    w.units = roff + M > 0 ? w.tiles_m * w.tiles_n : 0;
   }
   return w;
 }
@@ -176,13 +180,15 @@ __device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit&
 }
 
 // Issues this CTA's TMA loads of one stage; they complete on `cbar`, the even
-// CTA's full barrier (shared::cluster address).
+// CTA's full barrier (shared::cluster address). The dX GEMM's dZ rows start at
+// `roff`.
 template <int KIND>
 __device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMap* ma,
                                            const CUtensorMap* mb, uint32_t sa, uint32_t sb,
                                            uint32_t cbar, const Unit& t, int32_t kb,
-                                           uint32_t rank) {
-  const int32_t a0 = t.m_blk * kPairM + (int32_t)rank * kBM;
+                                           uint32_t rank, int64_t roff) {
+  const int32_t a0 =
+      t.m_blk * kPairM + (int32_t)rank * kBM + (KIND == GEMM_DX ? (int32_t)roff : 0);
   const int32_t b0 = t.n_blk * kBN + (int32_t)rank * kBNHalf;
   if (!Majors<KIND>::a_mn) {
     tma_load_2d_pair(sa, ma, cbar, kb * kBK, a0);
@@ -306,10 +312,10 @@ __device__ __forceinline__ void epi_fwd(const GemmParams& p, const CUtensorMap* 
 
 // GEMM_DZ: dz_{r,v} = w_r (1[v = y_r] - e^{z_{r,v} - lse_r}) as bf16, zero for
 // rows >= M and vocabulary columns >= V; 64-column sub-tiles leave through TMA
-// stores into dZ [m_pad, v_pad].
+// stores into dZ [dz_rows, v_pad], from row `roff` on.
 __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
-                                       const Unit& t, int64_t row0, int lane, uint32_t tb,
-                                       EpiStage& st) {
+                                       const Unit& t, int64_t row0, int64_t roff, int lane,
+                                       uint32_t tb, EpiStage& st) {
   const int64_t r = row0 + lane;
   const bool valid = r < M;
   float w = 0.f, lse_l2 = 0.f;
@@ -353,7 +359,8 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
     }
     const uint32_t sbuf = st.acquire(lane);
     stage_row(sbuf, lane, chunk);
-    st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, col0, (int32_t)row0); });
+    st.release(lane, sbuf,
+               [&](uint32_t a) { tma_store_2d(map_c, a, col0, (int32_t)(row0 + roff)); });
   }
 }
 
@@ -477,7 +484,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     set_device_error(err, kStatusInvalidArg, kernel_id<KIND>() * 16 + 1);
   }
   if (!BGPO_IN_BOUNDS(err, M >= 0 && M <= p.g.m_cap, kernel_id<KIND>() * 16 + 9)) M = 0;
-  const Work wk = make_work<KIND>(p, M);
+  // first dZ / Xm^T row of this sample: nonzero only when it pairs with a
+  // pending sample (the masking set it; the forward does not use dZ)
+  const int64_t roff = KIND == GEMM_FWD ? 0 : row_offset(err[ERR_ROW_OFF], p.w.dz_rows, p.g.m_pad);
+  const Work wk = make_work<KIND>(p, M, roff);
+  if (KIND == GEMM_DW && blockIdx.x == 0 && threadIdx.x == 0) {
+    // a dW GEMM meant to complete a pair whose first sample is not pending
+    // adds this sample alone: the other sample's contribution is missing
+    if (p.pair_consume && err[ERR_PAIRED] != 1)
+      set_device_error(err, kStatusInvalidArg, kernel_id<KIND>() * 16 + 5);
+    err[ERR_PEND] = -1;  // nothing waits any more
+  }
   // the split reduction after the dX GEMM reads the split count from here
   if (KIND == GEMM_DX && blockIdx.x == 0 && threadIdx.x == 0) err[ERR_DX_SPLITS] = wk.splits;
   if (pair >= wk.units) return;  // both CTAs of the pair, before any allocation
@@ -529,7 +546,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t cbar = map_to_cta(smem_addr(&full[stage]), 0);
           if (rank == 0) mbar_arrive_expect_tx(smem_addr(&full[stage]), bytes);
           load_stage<KIND>(p, &map_a, &map_b, smem_addr(s_a + stage * kTileABytes),
-                           smem_addr(s_b + stage * kTileBBytes), cbar, t, kb, rank);
+                           smem_addr(s_b + stage * kTileBBytes), cbar, t, kb, rank, roff);
           issued = true;
           if (++stage == kSt) { stage = 0; phase ^= 1u; }
         }
@@ -611,7 +628,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const uint32_t tb = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN);
       const int64_t row0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM + quarter * 32;
       if (KIND == GEMM_FWD) epi_fwd(p, &map_c, M, t, row0, lane, tb, st);
-      else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, lane, tb, st);
+      else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, roff, lane, tb, st);
       else if (KIND == GEMM_DX) epi_dx(p, &map_c, M, wk, t, row0, lane, tb, st);
       else epi_dw(p, &map_c, t, row0, lane, tb, st);
       tc_fence_before();
@@ -680,6 +697,7 @@ cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorM
   p.coef = a.coef;
   p.dW = a.dW;
   p.dX = a.dX;
+  p.pair_consume = a.pair_consume;
   switch (kind) {
     case GEMM_FWD: return launch_kind<GEMM_FWD>(map_a, map_b, map_c, p, s);
     case GEMM_DZ: return launch_kind<GEMM_DZ>(map_a, map_b, map_c, p, s);

@@ -119,6 +119,27 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
   if (tid == 0) {
     const int32_t M = s_carry;
     w.seg_off[a.B] = M;
+    // dW pairing: an odd sample pairs with sample j - 1 when that sample's
+    // backward left its rows pending in this workspace and no other sample has
+    // been masked here since (masking sample j again keeps the pairing). A
+    // pending sample that no pairing takes up would lose its dW contribution:
+    // that is an error, unless the pending sample itself is masked again (its
+    // backward will then run again).
+    const int32_t prev = w.err[ERR_SAMPLE];
+    const int32_t pend = w.err[ERR_PEND];
+    const bool pending = (pend & (int32_t)0xFFFF0000u) == pend_tag(0);
+    const int32_t pj = pend & 0xFFFF;
+    const bool paired = a.pair_dw && (a.j & 1) && pending && pj == a.j - 1 &&
+                        (prev == a.j - 1 || prev == a.j);
+    if (paired) {
+      w.err[ERR_ROW_OFF] = w.err[ERR_PEND_OFF];
+      w.err[ERR_PAIRED] = 1;
+    } else {
+      if (pending && pj != a.j) set_device_error(w.err, kStatusInvalidArg, KID_MASK_COMPACT * 16 + 5);
+      w.err[ERR_ROW_OFF] = 0;
+      w.err[ERR_PAIRED] = 0;
+      w.err[ERR_PEND] = -1;
+    }
     w.err[ERR_M] = M;
     w.err[ERR_SAMPLE] = a.j;
     w.err[ERR_LOGITS] = 0;  // no forward of this sample has kept its logits yet
@@ -229,7 +250,9 @@ __global__ void __launch_bounds__(kDzThreads, 4)
   const int64_t per_row = ceil_div(nvec, kDzItemVecs);
   const int64_t items = round_up(M, kPairM) * per_row;
   const float4* __restrict__ zc = reinterpret_cast<const float4*>(w.zc);
-  uint4* __restrict__ dz = reinterpret_cast<uint4*>(w.dz);
+  // this sample's dZ rows start at the pairing offset (0 without pairing)
+  uint4* __restrict__ dz = reinterpret_cast<uint4*>(w.dz) +
+                           row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad) * nvec;
   const int32_t V = (int32_t)g.V;
   for (int64_t q = blockIdx.x; q < items; q += gridDim.x) {
     const int64_t r = q / per_row;
@@ -379,9 +402,10 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
 }
 
 // ---------------------------------------------------------------------------
-// Xm^T [H, m_pad] from Xm [m_pad, H] for rows [0, round_up(M, 256)) of the
-// current sample (rows past M are the gather's zeros, so the K padding of the
-// dW GEMM reads zeros). With Xm^T the dW GEMM's B operand is K-major: one
+// Xm^T [H, dz_rows] from Xm [m_pad, H] for rows [0, round_up(M, 256)) of the
+// current sample, into columns [off, off + round_up(M, 256)) with off the
+// pairing offset (0 without pairing; rows past M are the gather's zeros, so the
+// K padding of the dW GEMM reads zeros). With Xm^T the dW GEMM's B operand is K-major: one
 // K-major and two MN-major boxes per stage instead of four MN-major boxes,
 // which measured 12% faster. 64 x 64 tiles through shared memory; 16-byte
 // global loads and stores; the row pitch of 66 elements keeps the column reads
@@ -390,9 +414,16 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
 constexpr int kTrTile = 64;
 constexpr int kTrPitch = kTrTile + 2;
 
-__global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, WsPtrs w) {
+__global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, bool defer,
+                                                      WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_XM_TRANSPOSE);
   if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_XM_TRANSPOSE * 16 + 9)) return;
+  const int64_t off = row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad);
+  if (defer && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) {
+    // the next sample's rows follow this sample's, from the next K block on
+    w.err[ERR_PEND_OFF] = (int32_t)round_up(M, kBK);
+    w.err[ERR_PEND] = pend_tag(j);
+  }
   const int64_t r0 = (int64_t)blockIdx.x * kTrTile;
   const int64_t h0 = (int64_t)blockIdx.y * kTrTile;
   if (r0 >= round_up(M, kPairM)) return;  // block-uniform
@@ -413,7 +444,7 @@ __global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, WsP
     for (int k = 0; k < 4; ++k)
       word[k] = (uint32_t)tile[(rr + 2 * k) * kTrPitch + hh] |
                 ((uint32_t)tile[(rr + 2 * k + 1) * kTrPitch + hh] << 16);
-    *reinterpret_cast<uint4*>(xmT + (h0 + hh) * g.m_pad + r0 + rr) =
+    *reinterpret_cast<uint4*>(xmT + (h0 + hh) * w.dz_rows + off + r0 + rr) =
         make_uint4(word[0], word[1], word[2], word[3]);
   }
 }
@@ -477,6 +508,7 @@ WsPtrs ws_pointers(void* ws, const WsLayout& L) {
   p.xm = base + L.xm;
   p.xmT = L.xmT ? base + L.xmT : nullptr;
   p.dz = base + L.dz;
+  p.dz_rows = (int64_t)L.dz_rows;
   p.dxp = reinterpret_cast<float*>(base + L.dxp);
   p.zc = L.zc_bytes ? reinterpret_cast<float*>(base + L.zc) : nullptr;
   return p;
@@ -539,9 +571,10 @@ cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, floa
   return cudaGetLastError();
 }
 
-cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, const WsPtrs& w, cudaStream_t s) {
+cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, bool defer, const WsPtrs& w,
+                                cudaStream_t s) {
   const dim3 grid((unsigned)(g.m_pad / kTrTile), (unsigned)(g.H / kTrTile));
-  k_xm_transpose<<<grid, 256, 0, s>>>(g, j, w);
+  k_xm_transpose<<<grid, 256, 0, s>>>(g, j, defer, w);
   return cudaGetLastError();
 }
 

@@ -45,12 +45,13 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None):
 
 
 def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None,
-            keep_logits=False):
+            keep_logits=False, pair_dw=False):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
     The old-policy pass is forward-only and keeps no logits; `keep_logits`
     sets BGPO_FLAG_KEEP_LOGITS for the inner loop (the workspace is sized for
-    it, and the old-policy pass runs on the same workspace without the flag).
+    it, and the old-policy pass runs on the same workspace without the flag);
+    `pair_dw` sets BGPO_FLAG_PAIR_DW for the inner loop in the same way.
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
     masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
@@ -62,7 +63,7 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     if resp_len is not None:
         lens = torch.as_tensor(np.asarray(resp_len), dtype=torch.int32, device=dev)
     prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                           resp_len=lens, keep_logits=keep_logits)
+                           resp_len=lens, keep_logits=keep_logits, pair_dw=pair_dw)
     prob_old = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
                                resp_len=lens)
     ws = bg.alloc_workspace(prob, dev)

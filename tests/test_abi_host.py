@@ -92,9 +92,10 @@ def test_validation_rejects_bad_offset_and_nonfinite_scale(L, bg):
 
 def test_validation_of_flags(L, bg):
     p = _prob(bg)
-    p.flags = bg.FLAG_KEEP_LOGITS
-    assert L.bgpo_validate_problem(ctypes.byref(p)) == 0
-    p.flags = 2                      # unknown bit
+    for f in (bg.FLAG_KEEP_LOGITS, bg.FLAG_PAIR_DW, bg.FLAG_KEEP_LOGITS | bg.FLAG_PAIR_DW):
+        p.flags = f
+        assert L.bgpo_validate_problem(ctypes.byref(p)) == 0
+    p.flags = 4                      # unknown bit
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
     p.flags = 0
@@ -113,9 +114,25 @@ def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
         assert keep - lean == -(-4 * m_pad * v_pad // 1024) * 1024
 
 
+def test_pairing_doubles_only_dz_and_xm_transpose(L, bg):
+    # BGPO_FLAG_PAIR_DW gives dZ [rows, roundup(V, 64)] and Xm^T [H, rows] twice
+    # the rows: 2 * roundup(B R, 256) * (roundup(V, 64) + H) more bytes, with or
+    # without the logit region
+    for (B, R, V, H) in ((2, 32, 512, 64), (3, 301, 1000, 192), (16, 512, 126464, 4096)):
+        m_pad = -(-B * R // 256) * 256
+        v_pad = -(-V // 64) * 64
+        for keep in (False, True):
+            lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep)))
+            pair = L.bgpo_workspace_bytes(ctypes.byref(
+                _prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep, pair_dw=True)))
+            assert pair - lean == 2 * m_pad * (v_pad + H)
+
+
 def test_workspace_independent_of_n_t(L, bg):
-    sizes = {n: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, n_t=n))) for n in (1, 2, 16, 32, 1000)}
-    assert len(set(sizes.values())) == 1 and sizes[1] > 0
+    for pair in (False, True):
+        sizes = {n: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, n_t=n, pair_dw=pair)))
+                 for n in (1, 2, 3, 16, 32, 1000)}
+        assert len(set(sizes.values())) == 1 and sizes[1] > 0
 
 
 def test_workspace_grows_with_rows_and_vocab(L, bg):
@@ -130,6 +147,8 @@ def test_workspace_of_paper_shapes_fits_hbm(L, bg):
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 3e9
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, keep_logits=True)
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
+    p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, pair_dw=True)
+    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 5e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5)
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 16e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5, keep_logits=True)

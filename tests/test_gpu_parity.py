@@ -400,14 +400,14 @@ def test_variable_length_responses(bg, keep):
     assert float(g["dX"][2, 117:].abs().max()) == 0.0
 
 
-@pytest.mark.parametrize("keep", [False, True])
-def test_whole_step_replays_from_a_cuda_graph(bg, keep):
-    # the n_t loop allocates nothing, never synchronises and keeps M on the
-    # device, so one step captures into a CUDA graph; a replay gives the bits
-    # of the eager step
+@pytest.mark.parametrize("keep,pair", [(False, False), (True, False), (False, True), (True, True)])
+def test_whole_step_replays_from_a_cuda_graph(bg, keep, pair):
+    # the n_t loop allocates nothing, never synchronises and keeps M (and the
+    # dW pairing state) on the device, so one step captures into a CUDA graph;
+    # a replay gives the bits of the eager step
     import torch
     wl, inp = _inputs("ragged")
-    p = bg.problem_from(wl, keep_logits=keep)
+    p = bg.problem_from(wl, keep_logits=keep, pair_dw=pair)
     X, W, Y = inp["X"], inp["W"], inp["Y"]
     ws = bg.alloc_workspace(p)
     A = inp["A"].contiguous()
@@ -469,9 +469,11 @@ def test_degenerate_shapes_match_oracle(bg, shape):
         assert float(g["ell"].abs().max()) <= 1e-4
 
 
-def test_peak_device_memory_flat_in_n_t(bg):
-    # Linearity (Sec. 3): one sample's state at a time, so the device memory a
-    # step needs does not grow with n_t; only the caller's [n_t, B] vectors do
+@pytest.mark.parametrize("pair", [False, True])
+def test_peak_device_memory_flat_in_n_t(bg, pair):
+    # Linearity (Sec. 3): one sample's state at a time (two with dW pairing), so
+    # the device memory a step needs does not grow with n_t; only the caller's
+    # [n_t, B] vectors do
     import torch
     peaks = {}
     for n_t in (1, 4, 16):
@@ -481,7 +483,7 @@ def test_peak_device_memory_flat_in_n_t(bg):
         torch.cuda.empty_cache()
         torch.cuda.reset_peak_memory_stats()
         base = torch.cuda.memory_allocated()
-        g = gpu_run(wl, inp)
+        g = gpu_run(wl, inp, pair_dw=pair)
         assert bg.get_device_error(g["ws"]) == (0, 0)
         peaks[n_t] = torch.cuda.max_memory_allocated() - base
         del g, inp
