@@ -40,20 +40,15 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind, from
-# the ncu capture of every GEMM launch of one llada8b_r512_b8 step (dW paired)
-# summarised in profiles/gemm_traffic_llada8b_r512_b8.md: affine fits in the
-# launch's rows (M, or K rows for dW). Valid only while the GEMM sources hash to
-# `sha`.
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind, mean
+# over one step of the bench workload with dW paired, from the single-pass ncu
+# capture summarised in profiles/gemm_traffic_llada8b_r512_onpolicy.md. Valid
+# only for that workload and mode, and while the GEMM sources hash to `sha`.
 TRAFFIC = {
-    "lmhead_fwd_lse": {"fixed_bytes": 1.0261e+09, "bytes_per_row": 30290.0,
-           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
-    "lmhead_dz": {"fixed_bytes": 9.8207e+08, "bytes_per_row": 356492.7,
-           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
-    "dx_gemm": {"fixed_bytes": 6.1442e+08, "bytes_per_row": 1290212.4,
-           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
-    "dw_gemm": {"fixed_bytes": 2.2937e+09, "bytes_per_row": 1220896.5,
-           "sha": "8c7ab10129b8221975cba1e0a42cd8ac923727ecd025c61b116e3f391b6cffce"},
+    "workload": "llada8b_r512_onpolicy",
+    "sha": "1a1434604d803d6abe19c88b879f873076a0becd35f6886ecc1866c0a15c6d01",
+    "bytes_per_launch": {"lmhead_fwd_lse": 2.1109e+09, "lmhead_dz": 3.8940e+09,
+                          "dx_gemm": 7.3817e+09, "dw_gemm": 1.4364e+10},
 }
 
 
@@ -372,8 +367,10 @@ def main():
     H, V = wl.H, wl.V
     gemm_flops_per_step = 2.0 * H * V * masked_per_step   # each GEMM kind of the step
 
-    def rooflines(per_kernel):
-        """Dominant GEMM against the sustained bf16 peak; the dz pass (if any) against HBM."""
+    def rooflines(per_kernel, headline_mode):
+        """Dominant GEMM against the sustained bf16 peak; the dz pass (if any) against HBM.
+        `headline_mode`: the leg runs the bench step (dW paired, logits recomputed),
+        the mode TRAFFIC was measured in."""
         gemm_kernels = [k for k in ("lmhead_fwd_lse", "lmhead_dz", "dx_gemm", "dw_gemm")
                         if k in per_kernel]
         dom = max(gemm_kernels, key=lambda k: per_kernel[k][1])
@@ -382,10 +379,9 @@ def main():
         dom_avg_s = dom_ms / dom_launches / 1e3
         achieved = dom_flops_per_launch / dom_avg_s / 1e12
         traffic = None
-        if dom in TRAFFIC and TRAFFIC[dom]["sha"] == kernel_sha():
-            # K rows of an average launch (two samples' rows when dW pairs them)
-            rows_per_launch = masked_per_step * args.steps / dom_launches
-            traffic = TRAFFIC[dom]["fixed_bytes"] + TRAFFIC[dom]["bytes_per_row"] * rows_per_launch
+        if (headline_mode and wl.name == TRAFFIC["workload"] and TRAFFIC["sha"] == kernel_sha()
+                and world == 1):
+            traffic = TRAFFIC["bytes_per_launch"].get(dom)
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
@@ -405,7 +401,7 @@ def main():
     # headline: logits recomputed in the backward, never stored; dW paired
     ms_local, per_kernel, clock_info, gpu_launches = timed_leg(False, pair, ws, True)
     ms, masked_all = aggregate_ranks(ms_local, masked_per_step)
-    roofline, _, n_gemm = rooflines(per_kernel)
+    roofline, _, n_gemm = rooflines(per_kernel, pair)
     value = masked_all / (ms / 1e3)
     exec_tflops = n_gemm * gemm_flops_per_step / (ms / 1e3) / 1e12
     useful_tflops = 3 * gemm_flops_per_step / (ms / 1e3) / 1e12   # fwd, dX, dW
@@ -435,7 +431,7 @@ def main():
     # the same step with the library's default flags (a dW GEMM per sample)
     if rank == 0 and world == 1 and pair:
         u_ms, u_per_kernel, _, u_launches = timed_leg(False, False, ws, False)
-        u_roof, _, _ = rooflines(u_per_kernel)
+        u_roof, _, _ = rooflines(u_per_kernel, False)
         out["unpaired"] = {
             "value": masked_per_step / (u_ms / 1e3), "unit": UNIT, "ms_per_step": u_ms,
             "gpu_launches": u_launches, "roofline": u_roof,
@@ -454,7 +450,7 @@ def main():
         ws_keep = bg.alloc_workspace(
             bg.problem_from(wl, b_offset=b_offset, keep_logits=True, pair_dw=pair), dev)
         k_ms, k_per_kernel, _, k_launches = timed_leg(True, pair, ws_keep, False)
-        k_roof, k_hbm, _ = rooflines(k_per_kernel)
+        k_roof, k_hbm, _ = rooflines(k_per_kernel, False)
         out["keep_logits"] = {
             "value": masked_per_step / (k_ms / 1e3), "unit": UNIT, "ms_per_step": k_ms,
             "gpu_launches": k_launches, "roofline": k_roof, "roofline_hbm_pass": k_hbm,
