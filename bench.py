@@ -46,9 +46,9 @@ UNIT = "tokens/s"
 # only for that workload and mode, and while the GEMM sources hash to `sha`.
 TRAFFIC = {
     "workload": "llada8b_r512_onpolicy",
-    "sha": "1a1434604d803d6abe19c88b879f873076a0becd35f6886ecc1866c0a15c6d01",
-    "bytes_per_launch": {"lmhead_fwd_lse": 2.1109e+09, "lmhead_dz": 3.8940e+09,
-                          "dx_gemm": 7.3817e+09, "dw_gemm": 1.4364e+10},
+    "sha": "10549a8464f33f9257c851e45de86d1a6ef464b6a5eb06635362b13a27d7693e",
+    "bytes_per_launch": {"lmhead_fwd_lse": 2.0363e+09, "lmhead_dz": 3.9066e+09,
+                          "dx_gemm": 7.5147e+09, "dw_gemm": 1.5873e+10},
 }
 
 

@@ -119,8 +119,10 @@ typedef struct bgpo_trace bgpo_trace;
  *       sample whose partner is not pending (its dW then holds sample j
  *       alone), or the masking of another sample while one is pending (the
  *       pending contribution is dropped). bgpo_clear_device_error forgets a
- *       pending sample. Keeping every sample's workspace apart (bgpo_vrpo_coeffs'
- *       "retain" strategy) does not pair: leave the flag off there.
+ *       pending sample. A repeated backward of the same odd sample adds that
+ *       sample's dW alone, as without the flag. Keeping every sample's
+ *       workspace apart (bgpo_vrpo_coeffs' "retain" strategy) does not pair:
+ *       leave the flag off there.
  */
 #define BGPO_FLAG_PAIR_DW 2u
 

@@ -185,9 +185,12 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits, bool pair_d
 //                 sample (ERR_PEND_OFF when it pairs with the pending sample,
 //                 else 0)
 //   ERR_PAIRED    set by the masking: 1 when the current sample pairs
+//   ERR_DW_K0     set by the backward before its dW GEMM: the first K row that
+//                 GEMM adds (0 while the partner is pending, ERR_ROW_OFF once
+//                 an earlier backward of this sample has added the partner)
 enum ErrField : int {
   ERR_STATUS = 0, ERR_WHERE = 1, ERR_SAMPLE = 2, ERR_M = 3, ERR_LOGITS = 4, ERR_DX_SPLITS = 5,
-  ERR_PEND = 6, ERR_PEND_OFF = 7, ERR_ROW_OFF = 8, ERR_PAIRED = 9
+  ERR_PEND = 6, ERR_PEND_OFF = 7, ERR_ROW_OFF = 8, ERR_PAIRED = 9, ERR_DW_K0 = 10
 };
 
 // Tag of a pending sample (n_t < 2^16): neither -1 nor a small integer that

@@ -64,6 +64,7 @@ struct GemmParams {
 
 struct Work {
   int64_t units, tiles_m, tiles_n, kb_total;
+  int64_t kb_first;  // first K block (dW: a partner already added is skipped)
   int splits;
 };
 
@@ -72,11 +73,14 @@ struct Unit {
 };
 
 // `roff`: the first dZ / Xm^T row of the sample (dW pairing; 0 otherwise). The
-// dW GEMM's K range [0, roff + M) then covers a pending sample's rows too.
+// dW GEMM's K range [k0, roff + M) then covers a pending sample's rows too when
+// k0 = 0.
 template <int KIND>
-__device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_t roff) {
+__device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_t roff,
+                                          int64_t k0) {
   Work w;
   w.splits = 1;
+  w.kb_first = 0;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
     w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = p.g.n_vt;
@@ -94,7 +98,8 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_
     w.tiles_m = ceil_div(p.g.V, kPairM);
     w.tiles_n = p.g.tiles_h;
     w.kb_total = ceil_div(roff + M, kBK);
-    w.units = roff + M > 0 ? w.tiles_m * w.tiles_n : 0;
+    w.kb_first = k0 / kBK;
+    w.units = w.kb_total > w.kb_first ? w.tiles_m * w.tiles_n : 0;
   }
   return w;
 }
@@ -125,8 +130,8 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
     // consecutive units share a vocabulary block of dZ^T
     t.m_blk = (int32_t)(u / w.tiles_n);
     t.n_blk = (int32_t)(u % w.tiles_n);
-    t.kb0 = 0;
-    t.kb_n = (int32_t)w.kb_total;
+    t.kb0 = (int32_t)w.kb_first;
+    t.kb_n = (int32_t)(w.kb_total - w.kb_first);
   }
   return t;
 }
@@ -487,7 +492,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   // first dZ / Xm^T row of this sample: nonzero only when it pairs with a
   // pending sample (the masking set it; the forward does not use dZ)
   const int64_t roff = KIND == GEMM_FWD ? 0 : row_offset(err[ERR_ROW_OFF], p.w.dz_rows, p.g.m_pad);
-  const Work wk = make_work<KIND>(p, M, roff);
+  // dW: first K row, a multiple of kBK in [0, roff] (see ERR_DW_K0)
+  const int64_t k0 = KIND == GEMM_DW ? row_offset(err[ERR_DW_K0], roff + p.g.m_pad, p.g.m_pad) : 0;
+  const Work wk = make_work<KIND>(p, M, roff, k0);
   if (KIND == GEMM_DW && blockIdx.x == 0 && threadIdx.x == 0) {
     // a dW GEMM meant to complete a pair whose first sample is not pending
     // adds this sample alone: the other sample's contribution is missing

@@ -419,10 +419,16 @@ __global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, boo
   const int32_t M = rows_of_sample(w.err, j, KID_XM_TRANSPOSE);
   if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_XM_TRANSPOSE * 16 + 9)) return;
   const int64_t off = row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad);
-  if (defer && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) {
-    // the next sample's rows follow this sample's, from the next K block on
-    w.err[ERR_PEND_OFF] = (int32_t)round_up(M, kBK);
-    w.err[ERR_PEND] = pend_tag(j);
+  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) {
+    // the dW GEMM after this kernel adds the pending partner's rows [0, off)
+    // only while the partner is still pending (a repeated backward of this
+    // sample adds its own rows alone)
+    w.err[ERR_DW_K0] = (w.err[ERR_PEND] == pend_tag(j - 1)) ? 0 : (int32_t)off;
+    if (defer) {
+      // the next sample's rows follow this sample's, from the next K block on
+      w.err[ERR_PEND_OFF] = (int32_t)round_up(M, kBK);
+      w.err[ERR_PEND] = pend_tag(j);
+    }
   }
   const int64_t r0 = (int64_t)blockIdx.x * kTrTile;
   const int64_t h0 = (int64_t)blockIdx.y * kTrTile;

@@ -160,3 +160,24 @@ def test_masking_a_sample_twice_keeps_the_pairing(bg):
         assert bg.get_device_error(ws) == (0, 0)
         outs.append((dX, dW))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_repeated_backward_adds_what_the_unpaired_path_adds(bg):
+    """Backward calls 0, 1, 1: the second call of sample 1 adds sample 1's dW
+    alone (its partner was added by the first), as the unpaired path does."""
+    import torch
+    wl = CONFIGS["ragged"].with_(n_t=4)
+    inp = make_inputs(wl, device="cuda")
+    outs = []
+    for pair in (False, True):
+        p = bg.problem_from(wl, pair_dw=pair)
+        ws = bg.alloc_workspace(p)
+        dX, dW = _buffers(wl)
+        _sample(bg, p, 0, inp, ws, dX, dW)
+        _sample(bg, p, 1, inp, ws, dX, dW)
+        bg.elbo_bwd_accumulate(p, 1, inp["X"], inp["W"], inp["Y"],
+                               torch.full((wl.B,), -0.25, device="cuda"), ws, dX, dW)
+        assert bg.get_device_error(ws) == (0, 0)
+        outs.append((dX, dW))
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert normwise(to64(outs[1][1]), to64(outs[0][1])) <= ORDER_TOL
