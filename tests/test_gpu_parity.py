@@ -331,9 +331,11 @@ def test_backward_without_kept_logits_is_refused(bg):
     assert float(dW.abs().max()) > 0.0
 
 
-def test_sequence_shards_reproduce_the_full_batch(bg):
+@pytest.mark.parametrize("pair", [False, True])
+def test_sequence_shards_reproduce_the_full_batch(bg, pair):
     """Data-parallel decomposition on one device: two shards with b_offset give
-    the whole batch's draws and l, and their dW sum to the whole batch's dW."""
+    the whole batch's draws and l, and their dW sum to the whole batch's dW
+    (with and without dW pairing inside each shard)."""
     import torch
     # two groups of 3 Bernoulli rewards (both mixed at this seed): each shard
     # normalises its own group (Eq. 18)
@@ -348,7 +350,7 @@ def test_sequence_shards_reproduce_the_full_batch(bg):
         sub = {"X": inp["X"][sl].contiguous(), "W": inp["W"], "Y": inp["Y"][sl].contiguous(),
                "A": None, "rewards": inp["rewards"][sl].contiguous(),
                "eps": inp["eps"][sl].contiguous()}
-        parts.append(gpu_run(half, sub, b_offset=3 * k))
+        parts.append(gpu_run(half, sub, b_offset=3 * k, pair_dw=pair))
     assert torch.equal(torch.cat([p["masks"] for p in parts], dim=1), full["masks"])
     ell = torch.cat([p["ell"] for p in parts])
     assert torch.allclose(ell, full["ell"], rtol=1e-6, atol=1e-6)
@@ -379,15 +381,15 @@ def test_bounded_wait_times_out_and_context_survives(bg):
     assert torch.isfinite(ell).all()
 
 
-@pytest.mark.parametrize("keep", [False, True])
-def test_variable_length_responses(bg, keep):
+@pytest.mark.parametrize("keep,pair", [(False, False), (True, False), (False, True)])
+def test_variable_length_responses(bg, keep, pair):
     """Padded batches: positions at or past resp_len[b] are never masked and get
     no gradient; everything else matches the oracle on the same draws (both
-    logit modes)."""
+    logit modes, and with dW pairing)."""
     wl = CONFIGS["ragged"]
     inp = make_inputs(wl, device="cuda")
     lens = np.array([301, 0, 117])
-    g = gpu_run(wl, inp, resp_len=lens, keep_logits=keep)
+    g = gpu_run(wl, inp, resp_len=lens, keep_logits=keep, pair_dw=pair)
     o = oracle_run(wl, {k: (v.cpu() if v is not None else None) for k, v in inp.items()},
                    resp_len=lens)
     assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
