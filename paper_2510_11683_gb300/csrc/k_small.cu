@@ -405,9 +405,9 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
 // Xm^T [H, dz_rows] from Xm [m_pad, H] for rows [0, round_up(M, 256)) of the
 // current sample, into columns [off, off + round_up(M, 256)) with off the
 // pairing offset (0 without pairing; rows past M are the gather's zeros, so the
-// K padding of the dW GEMM reads zeros). With Xm^T the dW GEMM's B operand is K-major: one
-// K-major and two MN-major boxes per stage instead of four MN-major boxes,
-// which measured 12% faster. 64 x 64 tiles through shared memory; 16-byte
+// K padding of the dW GEMM reads zeros). With Xm^T the dW GEMM's B operand is
+// K-major: one K-major and two MN-major boxes per stage instead of four
+// MN-major boxes, which measured 12% faster. 64 x 64 tiles through shared memory; 16-byte
 // global loads and stores; the row pitch of 66 elements keeps the column reads
 // to two-way bank conflicts.
 // ---------------------------------------------------------------------------
@@ -423,7 +423,7 @@ __global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, boo
     // the dW GEMM after this kernel adds the pending partner's rows [0, off)
     // only while the partner is still pending (a repeated backward of this
     // sample adds its own rows alone)
-    w.err[ERR_DW_K0] = (w.err[ERR_PEND] == pend_tag(j - 1)) ? 0 : (int32_t)off;
+    w.err[ERR_DW_K0] = (j > 0 && w.err[ERR_PEND] == pend_tag(j - 1)) ? 0 : (int32_t)off;
     if (defer) {
       // the next sample's rows follow this sample's, from the next K block on
       w.err[ERR_PEND_OFF] = (int32_t)round_up(M, kBK);

@@ -2,7 +2,8 @@
 
   * V = 2^24 - 1000 (just under the largest vocabulary, ragged against every
     tile width): 65,532 vocabulary tiles in the forward and dW GEMMs, a 2^24-long
-    K loop in the dX GEMM, 64-bit offsets into dZ and the kept logits;
+    K loop in the dX GEMM, 64-bit offsets into dZ and the kept logits, and into
+    the paired dZ rows with BGPO_FLAG_PAIR_DW;
   * B * R = 2^22 (the most response positions): the single-CTA mask compaction
     walks 2^20 Philox blocks, about 2^21 masked rows per sample;
   * H = 16384 (the largest hidden size): 64 hidden-size tiles, 256 K blocks per
@@ -56,8 +57,15 @@ def test_largest_vocabulary(bg):
     assert bg.get_device_error(k["ws"]) == (0, 0)
     assert torch.equal(k["ell"], g["ell"]) and torch.equal(k["dX"], g["dX"])
     assert torch.equal(k["dW"], g["dW"])
+    del k
+    # dW pairing puts sample 1's dZ rows after sample 0's (64-bit row offsets
+    # into a 2 * 256 x 2^24 bf16 region): same l and dX bits, dW up to order
+    q = gpu_run(wl, inp, pair_dw=True)
+    assert bg.get_device_error(q["ws"]) == (0, 0)
+    assert torch.equal(q["ell"], g["ell"]) and torch.equal(q["dX"], g["dX"])
+    assert normwise(to64(q["dW"]), to64(g["dW"])) <= 1e-5
     g = {key: g[key].cpu() for key in ("masks", "t", "ell", "dX", "dW")}
-    del k, inp
+    del q, inp
     torch.cuda.empty_cache()
     _check(wl, g, oracle_run(wl, inp_cpu))
 
