@@ -40,7 +40,8 @@
  *        bgpo_elbo_bwd_accumulate
  *    on one stream, with the same j. A call made with a j other than the one
  *    the workspace holds sets the device error word to BGPO_ERR_INVALID_ARG
- *    and does no work.
+ *    and does no work. With BGPO_FLAG_PAIR_DW the workspace also carries an
+ *    even sample's dL/dz rows into the next sample's backward (see the flag).
  *  - Host-side checks return a status before anything is launched. A failed
  *    launch returns BGPO_ERR_CUDA. Faults detected on the device (a non-finite
  *    coefficient, a bounded wait that ran out, a sample mismatch) are recorded
