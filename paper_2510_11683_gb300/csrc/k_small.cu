@@ -166,7 +166,16 @@ __global__ void __launch_bounds__(256) k_gather(Geometry g, int32_t j, const uin
     if (!BGPO_IN_BOUNDS(w.err, idx >= 0 && idx < g.m_cap, KID_GATHER * 16 + 10)) return;
     const int64_t b = idx / g.R, i = idx % g.R;
     const uint4* src = X + (b * (g.P + g.R) + g.P + i) * nvec;
-    for (int64_t v = lane; v < nvec; v += 32) dst[v] = __ldg(src + v);
+    // 8 loads of 16 bytes in flight per lane before their stores
+    for (int64_t v0 = lane; v0 < nvec; v0 += 32 * 8) {
+      uint4 q[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (v0 + 32 * k < nvec) q[k] = __ldg(src + v0 + 32 * k);
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (v0 + 32 * k < nvec) dst[v0 + 32 * k] = q[k];
+    }
     if (lane == 0) {
       const int32_t y = __ldg(Y + idx);
       (void)BGPO_IN_BOUNDS(w.err, y >= 0 && y < g.V, KID_GATHER * 16 + 11);  // a target outside V
@@ -187,6 +196,8 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
   else        { s = s + s2 * expf(m2 - m); }
 }
 
+constexpr int kLseBatch = 8;
+
 // ---------------------------------------------------------------------------
 // log-sum-exp of each masked row from the per-vocab-tile partials, then
 // log p(y_r) = z_{r, y_r} - lse_r. One warp per row, fixed merge order.
@@ -201,9 +212,17 @@ __global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, bool
   if (r >= M) return;
   float m = -INFINITY, s = 0.f;
   const float2* part = w.part + r * g.n_vt;
-  for (int64_t i = lane; i < g.n_vt; i += 32) {
-    const float2 p = part[i];
-    lse_merge(m, s, p.x, p.y);
+  // each lane merges partials lane, lane + 32, ... in order; kLseBatch loads
+  // are in flight before the merges that need them
+  for (int64_t i = lane; i < g.n_vt; i += 32 * kLseBatch) {
+    float2 q[kLseBatch];
+#pragma unroll
+    for (int k = 0; k < kLseBatch; ++k) {
+      const int64_t idx = i + 32 * k;
+      q[k] = idx < g.n_vt ? part[idx] : make_float2(-INFINITY, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < kLseBatch; ++k) lse_merge(m, s, q[k].x, q[k].y);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -407,15 +426,19 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
 // pairing offset (0 without pairing; rows past M are the gather's zeros, so the
 // K padding of the dW GEMM reads zeros). With Xm^T the dW GEMM's B operand is
 // K-major: one K-major and two MN-major boxes per stage instead of four
-// MN-major boxes, which measured 12% faster. 64 x 64 tiles through shared memory; 16-byte
-// global loads and stores; the row pitch of 66 elements keeps the column reads
-// to two-way bank conflicts.
+// MN-major boxes, which measured 12% faster. A block moves a 256-row x
+// 64-column tile through shared memory with 16-byte global loads and stores,
+// all 8 of a thread's loads in flight at once; the row pitch of 66 elements
+// keeps the column reads to two-way bank conflicts.
 // ---------------------------------------------------------------------------
-constexpr int kTrTile = 64;
-constexpr int kTrPitch = kTrTile + 2;
+constexpr int kTrRows = kPairM;   // one pair tile of rows per block
+constexpr int kTrCols = 64;
+constexpr int kTrPitch = kTrCols + 2;
+constexpr int kTrThreads = 256;
+constexpr int kTrChunks = kTrRows * kTrCols / 8 / kTrThreads;   // 16-byte chunks per thread
 
-__global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, bool defer,
-                                                      WsPtrs w) {
+__global__ void __launch_bounds__(kTrThreads) k_xm_transpose(Geometry g, int32_t j, bool defer,
+                                                             WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_XM_TRANSPOSE);
   if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_XM_TRANSPOSE * 16 + 9)) return;
   const int64_t off = row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad);
@@ -430,21 +453,32 @@ __global__ void __launch_bounds__(256) k_xm_transpose(Geometry g, int32_t j, boo
       w.err[ERR_PEND] = pend_tag(j);
     }
   }
-  const int64_t r0 = (int64_t)blockIdx.x * kTrTile;
-  const int64_t h0 = (int64_t)blockIdx.y * kTrTile;
+  const int64_t r0 = (int64_t)blockIdx.x * kTrRows;
+  const int64_t h0 = (int64_t)blockIdx.y * kTrCols;
   if (r0 >= round_up(M, kPairM)) return;  // block-uniform
-  __shared__ __align__(16) uint16_t tile[kTrTile * kTrPitch];
+  __shared__ __align__(16) uint16_t tile[kTrRows * kTrPitch];
   const uint16_t* __restrict__ xm = static_cast<const uint16_t*>(w.xm);
   uint16_t* __restrict__ xmT = static_cast<uint16_t*>(w.xmT);
-  for (int c = threadIdx.x; c < kTrTile * kTrTile / 8; c += blockDim.x) {
-    const int rr = c / 8, cc = (c % 8) * 8;
-    const uint4 v = *reinterpret_cast<const uint4*>(xm + (r0 + rr) * g.H + h0 + cc);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(tile + rr * kTrPitch + cc);
-    dst[0] = v.x; dst[1] = v.y; dst[2] = v.z; dst[3] = v.w;
+  uint4 v[kTrChunks];
+#pragma unroll
+  for (int i = 0; i < kTrChunks; ++i) {   // chunk c: row c / 8, columns (c % 8) * 8 ..
+    const int c = threadIdx.x + i * kTrThreads;
+    v[i] = *reinterpret_cast<const uint4*>(xm + (r0 + c / 8) * g.H + h0 + (c % 8) * 8);
+  }
+#pragma unroll
+  for (int i = 0; i < kTrChunks; ++i) {
+    const int c = threadIdx.x + i * kTrThreads;
+    uint32_t* dst = reinterpret_cast<uint32_t*>(tile + (c / 8) * kTrPitch + (c % 8) * 8);
+    dst[0] = v[i].x; dst[1] = v[i].y; dst[2] = v[i].z; dst[3] = v[i].w;
   }
   __syncthreads();
-  for (int c = threadIdx.x; c < kTrTile * kTrTile / 8; c += blockDim.x) {
-    const int hh = c / 8, rr = (c % 8) * 8;
+#pragma unroll
+  for (int i = 0; i < kTrChunks; ++i) {
+    // output chunk c: column hh of the tile, 8 rows from rr; 8 consecutive
+    // threads write one 128-byte segment of an Xm^T row
+    const int c = threadIdx.x + i * kTrThreads;
+    const int hh = (c / 8) % kTrCols;
+    const int rr = (c / (8 * kTrCols)) * 64 + (c % 8) * 8;
     uint32_t word[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
@@ -579,8 +613,8 @@ cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, floa
 
 cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, bool defer, const WsPtrs& w,
                                 cudaStream_t s) {
-  const dim3 grid((unsigned)(g.m_pad / kTrTile), (unsigned)(g.H / kTrTile));
-  k_xm_transpose<<<grid, 256, 0, s>>>(g, j, defer, w);
+  const dim3 grid((unsigned)(g.m_pad / kTrRows), (unsigned)(g.H / kTrCols));
+  k_xm_transpose<<<grid, kTrThreads, 0, s>>>(g, j, defer, w);
   return cudaGetLastError();
 }
 
