@@ -90,4 +90,9 @@ def test_largest_hidden_size(bg):
     inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
     g = gpu_run(wl, inp)
     assert bg.get_device_error(g["ws"]) == (0, 0)
-    _check(wl, g, oracle_run(wl, inp_cpu))
+    o = oracle_run(wl, inp_cpu)
+    _check(wl, g, o)
+    # dW pairing at the widest Xm^T rows (64 hidden-size tiles of the dW GEMM)
+    q = gpu_run(wl, inp, pair_dw=True)
+    assert bg.get_device_error(q["ws"]) == (0, 0)
+    _check(wl, q, o)
