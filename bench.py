@@ -41,9 +41,9 @@ METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind, mean
-# over one step of the bench workload with dW paired, from the single-pass ncu
-# capture summarised in profiles/gemm_traffic_llada8b_r512_onpolicy.md. Valid
-# only for that workload and mode, and while the GEMM sources hash to `sha`.
+# over one step of the bench workload with dW paired, from one single-pass ncu
+# capture of that step. Valid only for that workload and mode, and while the
+# GEMM sources hash to `sha` (otherwise the line reports traffic as null).
 TRAFFIC = {
     "workload": "llada8b_r512_onpolicy",
     "sha": "10549a8464f33f9257c851e45de86d1a6ef464b6a5eb06635362b13a27d7693e",

@@ -303,14 +303,19 @@ bgpo_status bgpo_group_advantage(const bgpo_problem* prob, const float* rewards,
  * need.
  *   X, W, Y   as for bgpo_elbo_fwd;  t_out device float [B] or NULL;
  *   ell_out   device float [B]: l_{b,j} (Eq. 4), same values as bgpo_elbo_fwd.
- * It keeps no logits (prob->flags is validated, then ignored).
+ * It keeps no logits (prob->flags is validated, then ignored). prob->resp_len,
+ * when given, must be 4-byte aligned like the other int32 pointers
+ * (BGPO_ERR_ALIGNMENT otherwise, before anything is launched).
  * Limit: the forward scratch of `prob` must fit the 32 MiB array, about
- * roundup(B*R, 128) * (2 H + 8 ceil(V / 256) + 20) bytes; larger problems
- * return BGPO_ERR_WORKSPACE_TOO_SMALL before anything is launched.
- * Every GPU that loads the library holds the 32 MiB until the process exits.
- * The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current); that first call should
- * come before any stream capture. Calls allocate nothing and free nothing.
+ * roundup(B*R, 256) * (2 H + 8 ceil(V / 256) + 20) + 16 B + 12288 bytes;
+ * larger problems return BGPO_ERR_WORKSPACE_TOO_SMALL before anything is
+ * launched. Every GPU that loads the library holds the 32 MiB until the
+ * process exits. The first call on each device looks up the array's device
+ * address (cudaGetSymbolAddress, with that device current) and caches it with
+ * the id of the current CUDA context; a call that finds another context
+ * current (after cudaDeviceReset, say) looks it up again. That first call
+ * should come before any stream capture. Calls allocate nothing and free
+ * nothing.
  * All calls share the one array, which keeps the previous call's contents:
  * calls whose GPU work overlaps (other streams, other host threads) race and
  * give undefined results. Device-side errors are recorded in the array's own

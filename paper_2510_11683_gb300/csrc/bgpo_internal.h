@@ -29,7 +29,9 @@ struct WsPtrs {
   float* zc;  // fp32 logits kept by the forward; null when the layout has none
 };
 
-WsPtrs ws_pointers(void* ws, const WsLayout& L);
+// `forward_only`: the buffer holds only the regions below L.fwd_bytes; the
+// backward regions (xmT, dz, dxp, zc) are given as null pointers.
+WsPtrs ws_pointers(void* ws, const WsLayout& L, bool forward_only = false);
 
 struct MaskArgs {
   uint64_t seed;

@@ -14,10 +14,12 @@
 // library holds kNoAllocScratchBytes of it until the process exits. Host code
 // cannot use the array's name as a device address, so the first call on each
 // device looks the address up with cudaGetSymbolAddress (with that device
-// current) and caches it; that first call should come before any stream
-// capture. All calls share the one array and it keeps the previous call's
-// contents, so calls whose GPU work overlaps (two streams, two host threads)
-// race on it.
+// current) and caches it together with the id of the CUDA context it belongs
+// to; a call that finds another context current (after cudaDeviceReset, for
+// instance, the module and its array are loaded again, possibly elsewhere)
+// looks it up again. That first call should come before any stream capture.
+// All calls share the one array and it keeps the previous call's contents, so
+// calls whose GPU work overlaps (two streams, two host threads) race on it.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -43,9 +45,42 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 namespace {
 
 std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxDevices];  // device address of g_noalloc_scratch, per device
+void* g_scratch_addr[kMaxDevices];              // device address of g_noalloc_scratch, per device
+unsigned long long g_scratch_ctx[kMaxDevices];  // id of the context that address belongs to
 
-// Device address of the scratch array on the current device (looked up once).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Id of the current CUDA context (0 when none is current or it cannot be read).
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(f);
+    else
+      cudaGetLastError();
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(f);
+    else
+      cudaGetLastError();
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current && get_id && get_current(&ctx) == CUDA_SUCCESS && ctx &&
+      get_id(ctx, &id) == CUDA_SUCCESS)
+    return id;
+  return 0;
+}
+
+// Device address of the scratch array on the current device, looked up once
+// per device and CUDA context.
 bgpo_status scratch_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) {
@@ -54,50 +89,21 @@ bgpo_status scratch_address(void** out) {
   }
   if (dev < 0 || dev >= kMaxDevices) return BGPO_ERR_UNSUPPORTED_DEVICE;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
+  const unsigned long long ctx = current_context_id();
+  if (!g_scratch_addr[dev] || ctx == 0 || ctx != g_scratch_ctx[dev]) {
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess || !p) {
       cudaGetLastError();
+      g_scratch_addr[dev] = nullptr;
       return BGPO_ERR_CUDA;
     }
     g_scratch_addr[dev] = p;
+    // the lookup makes the device's context current if none was
+    g_scratch_ctx[dev] = current_context_id();
   }
   *out = g_scratch_addr[dev];
   return BGPO_OK;
-}
-
-// Forward-only part of the workspace layout (no dZ / dX-partial regions).
-struct FwdLayout {
-  WsLayout L;
-  size_t total;
-};
-
-FwdLayout forward_layout(const Geometry& g) {
-  FwdLayout f;
-  WsLayout& L = f.L;
-  size_t o = 0;
-  L.err = o;       o = align_ws(o + 64);
-  L.t = o;         o = align_ws(o + 4 * (size_t)g.B);
-  L.tnum = o;      o = align_ws(o + 8 * (size_t)g.B);
-  L.seg_off = o;   o = align_ws(o + 4 * (size_t)(g.B + 1));
-  L.rows = o;      o = align_ws(o + 4 * (size_t)g.m_cap);
-  L.tgt = o;       o = align_ws(o + 4 * (size_t)g.m_pad);
-  L.tgt_logit = o; o = align_ws(o + 4 * (size_t)g.m_pad);
-  L.lse = o;       o = align_ws(o + 4 * (size_t)g.m_pad);
-  L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
-  L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
-  L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
-  L.xmT = 0;       // forward only
-  L.dz = 0;
-  L.dz_rows = (size_t)g.m_pad;
-  L.dxp = 0;
-  L.dxp_elems = 0;
-  L.zc = 0;        // keeps no logits
-  L.zc_bytes = 0;
-  L.total = o;
-  f.total = o;
-  return f;
 }
 
 bool encode_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
@@ -140,11 +146,13 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   if (j < 0 || j >= prob->n_t) return BGPO_ERR_INVALID_ARG;
   if (!X || !W || !Y || !ell_out) return BGPO_ERR_INVALID_ARG;
   if (!aligned_to(X, 16) || !aligned_to(W, 16) || !aligned_to(Y, 4) || !aligned_to(ell_out, 4) ||
-      (t_out && !aligned_to(t_out, 4)))
+      (t_out && !aligned_to(t_out, 4)) || (prob->resp_len && !aligned_to(prob->resp_len, 4)))
     return BGPO_ERR_ALIGNMENT;
   const Geometry g = make_geometry(prob->B, prob->P, prob->R, prob->H, prob->V);
-  const FwdLayout f = forward_layout(g);
-  if (f.total > kNoAllocScratchBytes) return BGPO_ERR_WORKSPACE_TOO_SMALL;
+  // the forward regions of the ordinary workspace layout (the same offsets
+  // under every flag); the backward regions do not exist here
+  const WsLayout L = make_ws_layout(g, false, false);
+  if (L.fwd_bytes > kNoAllocScratchBytes) return BGPO_ERR_WORKSPACE_TOO_SMALL;
 
   int dev = 0, major = 0, minor = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -160,7 +168,7 @@ extern "C" bgpo_status bgpo_elbo_fwd_noalloc(const bgpo_problem* prob, int32_t j
   if (st1 != BGPO_OK) return st1;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const WsPtrs w = ws_pointers(scratch, f.L);
+  const WsPtrs w = ws_pointers(scratch, L, /*forward_only=*/true);
   // The error word (status, where, sample tag, row count) must start at zero;
   // every other region is fully written before it is read within one call.
   if (cudaMemsetAsync(scratch, 0, 64, s) != cudaSuccess) {

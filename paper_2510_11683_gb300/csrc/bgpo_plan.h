@@ -118,6 +118,8 @@ struct WsLayout {
   size_t logp;       // float[m_pad] log p(y_r)
   size_t part;       // float2[m_pad * n_vt] (max, sum-exp) per (row, vocab tile)
   size_t xm;         // bf16[m_pad * H] gathered masked hidden states
+  size_t fwd_bytes;  // end of the regions a forward pass uses (err .. xm); the same under
+                     // every flag
   size_t xmT;        // bf16[H * dz_rows] the same, transposed (the dW GEMM's K-major operand)
   size_t dz;         // bf16[dz_rows * v_pad] dL/dz of the current sample (and of a pending one)
   size_t dz_rows;    // m_pad, or 2 m_pad when the dW GEMM pairs samples
@@ -159,6 +161,7 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits, bool pair_d
   L.logp = o;      o = align_ws(o + 4 * (size_t)g.m_pad);
   L.part = o;      o = align_ws(o + 8 * (size_t)g.m_pad * (size_t)g.n_vt);
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
+  L.fwd_bytes = o;
   L.xmT = o;       o = align_ws(o + 2 * (size_t)g.H * L.dz_rows);
   L.dz = o;        o = align_ws(o + 2 * L.dz_rows * (size_t)g.v_pad);
   L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;

@@ -532,7 +532,7 @@ cudaError_t launch_selftest_wait(int32_t* err, uint64_t timeout_ns, cudaStream_t
   return cudaGetLastError();
 }
 
-WsPtrs ws_pointers(void* ws, const WsLayout& L) {
+WsPtrs ws_pointers(void* ws, const WsLayout& L, bool forward_only) {
   char* base = static_cast<char*>(ws);
   WsPtrs p;
   p.err = reinterpret_cast<int32_t*>(base + L.err);
@@ -546,11 +546,11 @@ WsPtrs ws_pointers(void* ws, const WsLayout& L) {
   p.logp = reinterpret_cast<float*>(base + L.logp);
   p.part = reinterpret_cast<float2*>(base + L.part);
   p.xm = base + L.xm;
-  p.xmT = L.xmT ? base + L.xmT : nullptr;
-  p.dz = base + L.dz;
-  p.dz_rows = (int64_t)L.dz_rows;
-  p.dxp = reinterpret_cast<float*>(base + L.dxp);
-  p.zc = L.zc_bytes ? reinterpret_cast<float*>(base + L.zc) : nullptr;
+  p.xmT = forward_only ? nullptr : base + L.xmT;
+  p.dz = forward_only ? nullptr : base + L.dz;
+  p.dz_rows = forward_only ? 0 : (int64_t)L.dz_rows;
+  p.dxp = forward_only ? nullptr : reinterpret_cast<float*>(base + L.dxp);
+  p.zc = (!forward_only && L.zc_bytes) ? reinterpret_cast<float*>(base + L.zc) : nullptr;
   return p;
 }
 

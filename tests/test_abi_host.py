@@ -183,6 +183,20 @@ def test_null_and_misaligned_pointers(L, bg):
     assert L.bgpo_group_advantage(ctypes.byref(p), None, FAKE, None) == 1
 
 
+def test_noalloc_forward_validates_before_any_cuda_call(L, bg):
+    # bgpo_elbo_fwd_noalloc: every pointer check, including resp_len's
+    # alignment, returns before the library touches the device
+    p = _prob(bg)
+    t, ell = FAKE, FAKE
+    assert L.bgpo_elbo_fwd_noalloc(ctypes.byref(p), 0, None, FAKE, FAKE, t, ell, None) == 1
+    assert L.bgpo_elbo_fwd_noalloc(ctypes.byref(p), 0, FAKE + 8, FAKE, FAKE, t, ell, None) == 3
+    assert L.bgpo_elbo_fwd_noalloc(ctypes.byref(p), 0, FAKE, FAKE, FAKE, t + 2, ell, None) == 3
+    p.resp_len = FAKE + 2
+    assert L.bgpo_elbo_fwd_noalloc(ctypes.byref(p), 0, FAKE, FAKE, FAKE, t, ell, None) == 3
+    assert L.bgpo_sample_mask(ctypes.byref(p), 0, FAKE, L.bgpo_workspace_bytes(ctypes.byref(p)),
+                              None, None, None) == 3
+
+
 def test_workspace_too_small(L, bg):
     p = _prob(bg)
     ws = L.bgpo_workspace_bytes(ctypes.byref(p))

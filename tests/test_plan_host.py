@@ -30,11 +30,13 @@ static void layout(int64_t B, int64_t R, int64_t H, int64_t V) {
       printf("{\"kind\": \"layout\", \"B\": %lld, \"R\": %lld, \"H\": %lld, \"V\": %lld, "
              "\"keep\": %d, \"pair\": %d, \"off\": [%zu, %zu, %zu, %zu, %zu, %zu, %zu, %zu, %zu, "
              "%zu, %zu, %zu, %zu, %zu, %zu], \"dz_rows\": %zu, \"dxp_elems\": %zu, "
-             "\"zc_bytes\": %zu, \"total\": %zu, \"cap\": %lld}\n",
+             "\"zc_bytes\": %zu, \"total\": %zu, \"cap\": %lld, \"fwd\": %zu, \"m_pad\": %lld, "
+             "\"n_vt\": %lld}\n",
              (long long)B, (long long)R, (long long)H, (long long)V, keep, pair, L.err, L.t,
              L.tnum, L.seg_off, L.rows, L.tgt, L.tgt_logit, L.lse, L.logp, L.part, L.xm, L.xmT,
              L.dz, L.dxp, L.zc, L.dz_rows, L.dxp_elems, L.zc_bytes, L.total,
-             (long long)dxp_row_block_cap(g));
+             (long long)dxp_row_block_cap(g), L.fwd_bytes, (long long)g.m_pad,
+             (long long)g.n_vt);
     }
   const int64_t cap = dxp_row_block_cap(g);
   for (int64_t mb = 1; mb <= g.m_pad / kPairM; ++mb)
@@ -161,3 +163,15 @@ def test_pending_tags_are_not_small_integers(plan):
         tag = r["tag"]
         assert tag != -1 and not (0 <= tag < 65536), r
         assert (tag & 0xFFFF) == r["j"] and (tag >> 16) == 0x5EED, r
+
+
+def test_forward_regions_fit_the_documented_bound(plan):
+    # bgpo_elbo_fwd_noalloc needs the forward regions only; include/bgpo.h
+    # bounds them by roundup(B R, 256) (2 H + 8 ceil(V / 256) + 20) + 16 B + 12288
+    for L in plan["layout"]:
+        m_pad = -(-L["B"] * L["R"] // 256) * 256
+        assert L["m_pad"] == m_pad
+        bound = m_pad * (2 * L["H"] + 8 * -(-L["V"] // 256) + 20) + 16 * L["B"] + 12288
+        assert L["off"][10] < L["fwd"] <= bound           # xm starts below the end
+        assert L["fwd"] == L["off"][11]                    # Xm^T starts where it ends
+        assert L["fwd"] % 1024 == 0

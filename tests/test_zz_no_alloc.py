@@ -67,6 +67,9 @@ def test_noalloc_matches_workspace_path_on_two_calls_in_a_row(bg):
         assert torch.equal(t, t_ref)
         assert np.all(np.isfinite(ell.cpu().numpy()))
         assert rel_ell_err(ell.cpu().numpy(), ell_ref.cpu().numpy()).max() <= ELL_TOL
+        # the same kernels on the same inputs: stale scratch from the earlier,
+        # larger call must not change a single bit
+        assert torch.equal(ell, ell_ref)
 
 
 def test_noalloc_rejects_problems_beyond_its_scratch(bg):
@@ -79,3 +82,18 @@ def test_noalloc_rejects_problems_beyond_its_scratch(bg):
     ell = torch.zeros(wl.B, dtype=torch.float32, device="cuda")
     assert _noalloc(bg, prob, 0, x, x, y, None, ell) == 4   # BGPO_ERR_WORKSPACE_TOO_SMALL
     assert _noalloc(bg, bg.problem_from(CONFIGS["tiny"]), 9, x, x, y, None, ell) == 1
+
+
+def test_noalloc_rejects_a_misaligned_response_length_pointer(bg):
+    # a resp_len pointer that is not 4-byte aligned is refused on the host
+    # (BGPO_ERR_ALIGNMENT) before any kernel could load from it
+    import torch
+    wl = CONFIGS["tiny"]
+    inp = make_inputs(wl, device="cuda")
+    lens = torch.full((wl.B + 1,), wl.R, dtype=torch.int32, device="cuda")
+    raw = bg.problem_from(wl)
+    raw.resp_len = lens.data_ptr() + 2
+    ell = torch.full((wl.B,), float("nan"), device="cuda")
+    assert _noalloc(bg, raw, 0, inp["X"], inp["W"], inp["Y"], None, ell) == 3
+    torch.cuda.synchronize()
+    assert torch.isnan(ell).all()
