@@ -234,26 +234,30 @@ def group_advantage(rewards, G):
 # Gradients of one MC sample (backpropagation of L_j, Algorithm 1)
 # ---------------------------------------------------------------------------
 
-def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192):
+def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192, with_ell=False):
     """Gradient of sum_b coef_b * l_b (one MC sample) w.r.t. X and W.
 
     With w_r = coef_b / t_b for masked row r of sequence b and p_r = softmax(W x_r):
       dz_r = w_r (onehot(y_r) - p_r),  dX[b, i] = W^T dz_r,  dW = sum_r dz_r x_r^T.
     Returns (dX_resp [B, R, H], dW [V, H]) in fp64; dX covers response rows only
-    (prompt rows get no gradient from Eq. 4).
+    (prompt rows get no gradient from Eq. 4). with_ell=True also returns the
+    per-step ELBO term l [B] of Eq. 4 from the same log-probabilities, first:
+    (l, dX_resp, dW).
     """
     W = np.asarray(W, dtype=np.float64)
     B, R = mask.shape
     V, H = W.shape
     dX = np.zeros((B, R, H))
     dW = np.zeros((V, H))
+    ell = np.zeros(B)
     for b in range(B):
         idx = np.nonzero(mask[b])[0]
         if idx.size == 0:
             continue
         rows = response_rows(X, P, b, idx)
         y = np.asarray(Y[b, idx], dtype=np.int64)
-        _, lse = token_logprobs(rows, W, y, chunk)
+        logp, lse = token_logprobs(rows, W, y, chunk)
+        ell[b] = logp.sum() / t[b]
         w = coef[b] / t[b]
         for v0 in range(0, V, chunk):
             v1 = min(V, v0 + chunk)
@@ -263,6 +267,8 @@ def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192):
             dz[np.nonzero(hit)[0], y[hit] - v0] += w
             dW[v0:v1] += dz.T @ rows
             dX[b, idx] += dz @ W[v0:v1]
+    if with_ell:
+        return ell, dX, dW
     return dX, dW
 
 
@@ -306,6 +312,42 @@ def bgpo_step(X, W, Y, P, A, ell_old, ts, masks, loss_scale):
     R_lb = g.sum(axis=1)
     return dict(ell=ell, d=d, g=g, coef=coef, R_lb=R_lb,
                 loss=-loss_scale * R_lb.sum(), dX=dX, dW=dW)
+
+
+def bgpo_step_per_sample_x(Xs, W, Y, P, A, ell_old, ts, masks, loss_scale):
+    """Algorithm 1 with hidden states that differ between MC samples.
+
+    In the paper p_theta(y^i | y_t, x) conditions on the masked sequence y_t
+    (Sec. 2.1, Eq. 4), so every MC sample j runs the network on its own input
+    and its LM head sees its own final hidden states X_j. Xs [n_t, B, P+R, H]
+    holds X_j for each j. Each sample's l_j, bound coefficients (Eq. 10, 13) and
+    gradient are those of bgpo_step with X replaced by X_j; the gradient of
+    dHidden is per sample (it flows back through sample j's own forward pass),
+    while dW accumulates over the samples (Algorithm 1).
+    Returns dict: ell, d, g, coef [B, n_t], R_lb [B], loss, dX [n_t, B, R, H]
+    (dL/dX_j for each j), dW [V, H].
+    """
+    n_t = len(ts)
+    ell = np.stack([elbo_term(Xs[j], W, Y, P, masks[j], ts[j]) for j in range(n_t)], axis=1)
+    d, g, coef = bound_coeffs(ell, ell_old, np.asarray(A)[:, None], n_t, loss_scale)
+    B, R = masks.shape[1:]
+    V, H = np.asarray(W).shape
+    dX = np.zeros((n_t, B, R, H))
+    dW = np.zeros((V, H))
+    for j in range(n_t):   # gradient accumulation, one MC sample at a time
+        gx, gw = elbo_term_grads(Xs[j], W, Y, P, masks[j], ts[j], coef[:, j])
+        dX[j] = gx
+        dW += gw
+    R_lb = g.sum(axis=1)
+    return dict(ell=ell, d=d, g=g, coef=coef, R_lb=R_lb,
+                loss=-loss_scale * R_lb.sum(), dX=dX, dW=dW)
+
+
+def bgpo_loss_per_sample_x(Xs, W, Y, P, A, ell_old, ts, masks, loss_scale):
+    """Scalar loss of bgpo_step_per_sample_x with the draws held fixed."""
+    ell = np.stack([elbo_term(Xs[j], W, Y, P, masks[j], ts[j]) for j in range(len(ts))], axis=1)
+    _, g, _ = bound_coeffs(ell, ell_old, np.asarray(A)[:, None], len(ts), loss_scale)
+    return -loss_scale * g.sum()
 
 
 def bgpo_loss(X, W, Y, P, A, ell_old, ts, masks, loss_scale):

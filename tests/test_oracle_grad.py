@@ -162,3 +162,90 @@ def test_mc_gradient_std_shrinks_with_n_t():
             grads.append(O.bgpo_step(X, W, Y, P, A, ell, ts, masks, 1.0)["dW"])
         stds.append(O.grad_std_bias(np.stack(grads), np.zeros_like(W))[0])
     assert stds[0] > stds[1] > stds[2]
+
+
+def test_gradient_pass_returns_the_elbo_of_the_same_log_probabilities():
+    # with_ell: l of Eq. 4 from the gradient pass itself; closed form at W = 0
+    # (every log p = -log V) and equal to elbo_term otherwise
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=10, n_t=2)
+    coef = np.linspace(-1.0, 1.0, X.shape[0])
+    ell, gx, gw = O.elbo_term_grads(X, W, Y, P, masks[1], ts[1], coef, chunk=7, with_ell=True)
+    assert np.allclose(ell, O.elbo_term(X, W, Y, P, masks[1], ts[1]), rtol=1e-14, atol=0)
+    gx2, gw2 = O.elbo_term_grads(X, W, Y, P, masks[1], ts[1], coef, chunk=7)
+    assert np.array_equal(gx, gx2) and np.array_equal(gw, gw2)
+    Z = np.zeros_like(W)
+    ell0, _, _ = O.elbo_term_grads(X, Z, Y, P, masks[0], ts[0], coef, with_ell=True)
+    V = W.shape[0]
+    k = masks[0].sum(axis=1).astype(np.float64)
+    assert np.allclose(ell0, -k / ts[0] * np.log(V), rtol=1e-14, atol=0)
+
+
+def _per_sample_case(seed, n_t=3, **kw):
+    X, W, Y, P, A, _, ts, masks = _case(seed=seed, n_t=n_t, **kw)
+    rng = np.random.default_rng(seed + 50)
+    # each MC sample sees its own hidden states (Sec. 2.1: p_theta conditions on y_t)
+    Xs = np.stack([X + 0.5 * rng.standard_normal(X.shape) for _ in range(n_t)])
+    ell_self = np.stack([O.elbo_term(Xs[j], W, Y, P, masks[j], ts[j]) for j in range(n_t)], axis=1)
+    ell_old = ell_self + rng.standard_normal(ell_self.shape) * 0.3
+    return Xs, W, Y, P, A, ell_old, ts, masks
+
+
+def test_per_sample_hidden_states_match_finite_differences():
+    Xs, W, Y, P, A, ell_old, ts, masks = _per_sample_case(seed=11)
+    ls = 0.5
+    out = O.bgpo_step_per_sample_x(Xs, W, Y, P, A, ell_old, ts, masks, ls)
+    rng = np.random.default_rng(11)
+    h = 1e-6
+    f = lambda Xs_, W_: O.bgpo_loss_per_sample_x(Xs_, W_, Y, P, A, ell_old, ts, masks, ls)
+    n_t, B, R, H = out["dX"].shape
+    for _ in range(25):
+        j, b, i, k = rng.integers(n_t), rng.integers(B), rng.integers(R), rng.integers(H)
+        Xp, Xm = Xs.copy(), Xs.copy()
+        Xp[j, b, P + i, k] += h
+        Xm[j, b, P + i, k] -= h
+        fd = (f(Xp, W) - f(Xm, W)) / (2 * h)
+        assert abs(fd - out["dX"][j, b, i, k]) <= 1e-6 * max(1.0, abs(fd)), (j, b, i, k)
+    V = W.shape[0]
+    for _ in range(25):
+        v, k = rng.integers(V), rng.integers(H)
+        Wp, Wm = W.copy(), W.copy()
+        Wp[v, k] += h
+        Wm[v, k] -= h
+        fd = (f(Xs, Wp) - f(Xs, Wm)) / (2 * h)
+        assert abs(fd - out["dW"][v, k]) <= 1e-6 * max(1.0, abs(fd)), (v, k)
+
+
+def test_per_sample_hidden_states_match_torch_autograd():
+    # the loss restated with torch ops on a leaf tensor per MC sample's hidden states
+    Xs, W, Y, P, A, ell_old, ts, masks = _per_sample_case(seed=12, n_t=4, B=3, R=10, H=7, V=29)
+    ls = 0.25
+    out = O.bgpo_step_per_sample_x(Xs, W, Y, P, A, ell_old, ts, masks, ls)
+    Xt = torch.tensor(Xs, requires_grad=True)
+    Wt = torch.tensor(W, requires_grad=True)
+    n_t = len(ts)
+    total = torch.zeros((), dtype=torch.float64)
+    for j in range(n_t):
+        for b in range(Xs.shape[1]):
+            m = torch.from_numpy(masks[j, b].astype(bool))
+            z = Xt[j, b, P:] @ Wt.T
+            lp = torch.log_softmax(z, dim=1).gather(1, torch.from_numpy(Y[b]).long()[:, None])[:, 0]
+            ell = (lp * m).sum() / float(ts[j, b])
+            d = ell - float(ell_old[b, j])
+            g = (1 + d) * A[b] / n_t if A[b] >= 0 else torch.exp(d) * A[b] / n_t
+            total = total - ls * g
+    total.backward()
+    assert abs(float(total.detach()) - out["loss"]) < 1e-10 * max(1, abs(out["loss"]))
+    assert np.allclose(Wt.grad.numpy(), out["dW"], rtol=1e-10, atol=1e-12)
+    assert np.allclose(Xt.grad[:, :, P:].numpy(), out["dX"], rtol=1e-10, atol=1e-12)
+    assert not np.any(Xt.grad[:, :, :P].numpy())
+
+
+def test_shared_hidden_states_reduce_to_the_accumulated_step():
+    # the same X for every sample: per-sample dX_j sum to bgpo_step's accumulated dX
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=13, n_t=3)
+    Xs = np.stack([X] * 3)
+    a = O.bgpo_step_per_sample_x(Xs, W, Y, P, A, ell_old, ts, masks, 0.5)
+    b = O.bgpo_step(X, W, Y, P, A, ell_old, ts, masks, 0.5)
+    assert np.allclose(a["dX"].sum(axis=0), b["dX"], rtol=1e-12, atol=1e-14)
+    assert np.allclose(a["dW"], b["dW"], rtol=1e-12, atol=1e-14)
+    assert np.array_equal(a["ell"], b["ell"])
