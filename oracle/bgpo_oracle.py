@@ -116,11 +116,25 @@ def sample_t_mask_scalar(seed, B, R, j, n_t, t_mode):
 # LM head: log p_theta(y^i | y_t, x) = log_softmax(W x)[y^i]   (Eq. 4)
 # ---------------------------------------------------------------------------
 
-def token_logprobs(rows, W, y, chunk=8192):
+# Logit chunks of one sequence are kept between passes when they hold at most
+# this many elements (2 GiB of fp64); larger ones are recomputed per pass.
+Z_KEEP_ELEMS = 1 << 28
+
+
+def logit_chunks(rows, W, chunk=8192):
+    """z = W x_r for each row, as a list of [n, chunk] fp64 column blocks."""
+    rows = np.asarray(rows, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    return [rows @ W[v0:v0 + chunk].T for v0 in range(0, W.shape[0], chunk)]
+
+
+def token_logprobs(rows, W, y, chunk=8192, z_chunks=None):
     """log softmax(W x_r)[y_r] for each row x_r, in fp64, over vocab chunks.
 
     rows [n, H], W [V, H], y [n] -> (logp [n], lse [n]). The max shift is the
-    textbook one: lse = m + log sum exp(z - m).
+    textbook one: lse = m + log sum exp(z - m). z_chunks: the logits as
+    logit_chunks(rows, W, chunk) returns them, if already computed (otherwise
+    each pass computes them again).
     """
     rows = np.asarray(rows, dtype=np.float64)
     W = np.asarray(W, dtype=np.float64)
@@ -128,14 +142,16 @@ def token_logprobs(rows, W, y, chunk=8192):
     V = W.shape[0]
     if n == 0:
         return np.zeros(0), np.zeros(0)
+
+    def z_of(c, v0):
+        return z_chunks[c] if z_chunks is not None else rows @ W[v0:v0 + chunk].T
+
     m = np.full(n, -np.inf)
-    for v0 in range(0, V, chunk):
-        z = rows @ W[v0:v0 + chunk].T
-        m = np.maximum(m, z.max(axis=1))
+    for c, v0 in enumerate(range(0, V, chunk)):
+        m = np.maximum(m, z_of(c, v0).max(axis=1))
     s = np.zeros(n)
-    for v0 in range(0, V, chunk):
-        z = rows @ W[v0:v0 + chunk].T
-        s += np.exp(z - m[:, None]).sum(axis=1)
+    for c, v0 in enumerate(range(0, V, chunk)):
+        s += np.exp(z_of(c, v0) - m[:, None]).sum(axis=1)
     lse = m + np.log(s)
     z_y = np.einsum("nh,nh->n", rows, W[np.asarray(y, dtype=np.int64)])
     return z_y - lse, lse
@@ -256,12 +272,13 @@ def elbo_term_grads(X, W, Y, P, mask, t, coef, chunk=8192, with_ell=False):
             continue
         rows = response_rows(X, P, b, idx)
         y = np.asarray(Y[b, idx], dtype=np.int64)
-        logp, lse = token_logprobs(rows, W, y, chunk)
+        zs = logit_chunks(rows, W, chunk) if rows.shape[0] * V <= Z_KEEP_ELEMS else None
+        logp, lse = token_logprobs(rows, W, y, chunk, zs)
         ell[b] = logp.sum() / t[b]
         w = coef[b] / t[b]
-        for v0 in range(0, V, chunk):
+        for c, v0 in enumerate(range(0, V, chunk)):
             v1 = min(V, v0 + chunk)
-            z = rows @ W[v0:v1].T
+            z = zs[c] if zs is not None else rows @ W[v0:v1].T
             dz = -w * np.exp(z - lse[:, None])
             hit = (y >= v0) & (y < v1)
             dz[np.nonzero(hit)[0], y[hit] - v0] += w

@@ -119,3 +119,12 @@ def test_mc_elbo_estimate_converges():
     ell = O.elbo_all(X, W, Y, 0, ts, masks)[0]
     se = ell.std() / math.sqrt(n_t)
     assert abs(ell.mean() - exact) < 6 * se + 1e-9
+
+
+def test_logp_from_precomputed_logit_chunks():
+    X, W, Y = _tiny(B=1, P=0, R=30, H=12, V=100, seed=9, scale=2.0)
+    zs = O.logit_chunks(X[0], W, chunk=33)
+    assert [z.shape[1] for z in zs] == [33, 33, 33, 1]
+    a = O.token_logprobs(X[0], W, Y[0], chunk=33)
+    b = O.token_logprobs(X[0], W, Y[0], chunk=33, z_chunks=zs)
+    assert np.allclose(a[0], b[0], rtol=0, atol=1e-13) and np.allclose(a[1], b[1], rtol=0, atol=1e-13)

@@ -249,3 +249,15 @@ def test_shared_hidden_states_reduce_to_the_accumulated_step():
     assert np.allclose(a["dX"].sum(axis=0), b["dX"], rtol=1e-12, atol=1e-14)
     assert np.allclose(a["dW"], b["dW"], rtol=1e-12, atol=1e-14)
     assert np.array_equal(a["ell"], b["ell"])
+
+
+def test_kept_and_recomputed_logit_chunks_agree(monkeypatch):
+    # the gradient pass keeps each sequence's logit chunks between its passes
+    # when they are small; forcing the recompute path changes nothing
+    X, W, Y, P, A, ell_old, ts, masks = _case(seed=14, n_t=2, V=41)
+    coef = np.array([0.7, -1.3, 0.2])
+    kept = O.elbo_term_grads(X, W, Y, P, masks[1], ts[1], coef, chunk=6, with_ell=True)
+    monkeypatch.setattr(O, "Z_KEEP_ELEMS", 0)
+    again = O.elbo_term_grads(X, W, Y, P, masks[1], ts[1], coef, chunk=6, with_ell=True)
+    for a, b in zip(kept, again):
+        assert np.allclose(a, b, rtol=1e-14, atol=1e-15)
