@@ -141,3 +141,39 @@ def make_inputs(wl, device="cpu", need_w=True):
     if device != "cpu":
         out = {k: (v.to(device) if v is not None else None) for k, v in out.items()}
     return out
+
+
+def make_old_head(wl, W, delta=0.05):
+    """An old-policy LM head W_old = W + delta * N(0, 1/H), rounded to bf16.
+
+    Eq. 10 evaluates the current and the old policy on the same draws; a second
+    head makes the two policies' l differ through the model rather than through
+    a perturbation added to l. Seeded by (wl.seed, 0x01D); W is the bf16 head of
+    make_inputs (CPU or device; the result lands on W's device).
+    """
+    import torch
+
+    rng = np.random.default_rng([wl.seed, 0x01D])
+    noise = rng.standard_normal((wl.V, wl.H), dtype=np.float32) * np.float32(delta / np.sqrt(wl.H))
+    Wf = W.detach().to("cpu", torch.float32) + torch.from_numpy(noise)
+    return Wf.to(torch.bfloat16).to(W.device)
+
+
+def make_per_sample_hidden(wl, X, rho=0.8):
+    """Final hidden states that differ between MC samples: X_j [n_t, B, P+R, H].
+
+    In the paper each MC sample runs the network on its own masked sequence, so
+    its hidden states differ (Sec. 2.1). X_j = rho X + sqrt(1 - rho^2) N(0, 1),
+    drawn in fp32 from (wl.seed, 0x51, j) and rounded to bf16; X is the bf16
+    tensor of make_inputs (the result lands on X's device).
+    """
+    import torch
+
+    c = np.float32(np.sqrt(1.0 - rho * rho))
+    Xf = X.detach().to("cpu", torch.float32)
+    out = torch.empty((wl.n_t,) + tuple(X.shape), dtype=torch.bfloat16)
+    for j in range(wl.n_t):
+        rng = np.random.default_rng([wl.seed, 0x51, j])
+        z = rng.standard_normal(tuple(X.shape), dtype=np.float32)
+        out[j] = (Xf * np.float32(rho) + torch.from_numpy(z) * c).to(torch.bfloat16)
+    return out.to(X.device)

@@ -31,27 +31,46 @@ def oracle_advantages(wl, inp):
     return O.group_advantage(to64(inp["rewards"]), wl.G)
 
 
-def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None):
-    """Algorithm 1 inner loops in fp64: draws, l_self, l_old = l_self + eps, bound, grads."""
+def record_margin(test, **values):
+    """Appends one JSON line of parity margins (errors reached against the
+    oracle) to the file named by BGPO_MARGINS_OUT, when that is set."""
+    import json
+    import os
+    path = os.environ.get("BGPO_MARGINS_OUT")
+    if path:
+        with open(path, "a") as f:
+            f.write(json.dumps({"test": test, **{k: float(v) for k, v in values.items()}}) + "\n")
+
+
+def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None, W_old=None):
+    """Algorithm 1 inner loops in fp64: draws, l_self, l_old, bound, grads.
+
+    l_old = l_self + eps, or, with a second head W_old, the old policy's own
+    l on the same draws (Eq. 10)."""
     X, W, Y = to64(inp["X"]), to64(inp["W"]), to64(inp["Y"])
     ls = 1.0 / wl.G if loss_scale is None else loss_scale
     A = oracle_advantages(wl, inp)
     ts, masks = O.sample_masks(wl.seed, wl.B, wl.R, wl.n_t, wl.t_mode, b_offset, resp_len)
     ell_self = O.elbo_all(X, W, Y, wl.P, ts, masks)
-    ell_old = ell_self + to64(inp["eps"])
+    if W_old is None:
+        ell_old = ell_self + to64(inp["eps"])
+    else:
+        ell_old = O.elbo_all(X, to64(W_old), Y, wl.P, ts, masks)
     out = O.bgpo_step(X, W, Y, wl.P, A, ell_old, ts, masks, ls)
     out.update(ts=ts, masks=masks, A=A, ell_old=ell_old, ell_self=ell_self)
     return out
 
 
 def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None,
-            keep_logits=False, pair_dw=False):
+            keep_logits=False, pair_dw=False, W_old=None):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
     The old-policy pass is forward-only and keeps no logits; `keep_logits`
     sets BGPO_FLAG_KEEP_LOGITS for the inner loop (the workspace is sized for
     it, and the old-policy pass runs on the same workspace without the flag);
     `pair_dw` sets BGPO_FLAG_PAIR_DW for the inner loop in the same way.
+    W_old (device bf16 [V, H]): the old-policy pass runs with this head and
+    l_old is its output (no eps); otherwise l_old = l_self + eps.
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
     masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
@@ -80,8 +99,11 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     ell_self = torch.empty((n_t, B), dtype=torch.float32, device=dev)
     for j in range(n_t):          # old-policy pass (same draws, Eq. 10)
         bg.sample_mask(prob_old, j, ws, t[j], masks[j])
-        bg.elbo_fwd(prob_old, j, X, W, Y, ws, ell_self[j])
-    ell_old = (ell_self + inp["eps"].T.contiguous()).contiguous()
+        bg.elbo_fwd(prob_old, j, X, W if W_old is None else W_old, Y, ws, ell_self[j])
+    if W_old is None:
+        ell_old = (ell_self + inp["eps"].T.contiguous()).contiguous()
+    else:
+        ell_old = ell_self.clone()
     ell = torch.empty((n_t, B), dtype=torch.float32, device=dev)
     coef = torch.empty((n_t, B), dtype=torch.float32, device=dev)
     g = torch.empty((n_t, B), dtype=torch.float32, device=dev)
