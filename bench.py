@@ -18,9 +18,15 @@ fp64 oracle on a bounded sample of the same workload on the host cores.
 The step runs with BGPO_FLAG_PAIR_DW (MC samples 2k and 2k + 1 share one dW
 GEMM; the loop above is exactly the call order that flag expects) unless
 `--no-pair-dw` is given. `unpaired` = the same step without it (the library's
-default flags); `keep_logits` = the same step with BGPO_FLAG_KEEP_LOGITS too
-(the forward keeps its fp32 logits, the backward reads them instead of
-recomputing them).
+default flags: the backward walks the vocabulary in chunks of at most 32,768
+columns, so its dL/dz buffer holds one chunk); `unpaired_whole_vocab` = the
+unpaired step with the whole vocabulary as one chunk; `keep_logits` = the
+paired step with BGPO_FLAG_KEEP_LOGITS too (the forward keeps its fp32 logits,
+the backward reads them instead of recomputing them).
+
+Under torchrun (N > 1) every rank owns B responses of an N * B batch and each
+step ends with the one data-parallel exchange, the sum of dW over the ranks
+(paper_2510_11683_gb300.dp.allreduce_dw, NCCL), inside the timed region.
 """
 import argparse
 import hashlib
@@ -66,6 +72,8 @@ def parse():
                     help="skip the timed leg with BGPO_FLAG_KEEP_LOGITS")
     ap.add_argument("--no-pair-dw", action="store_true",
                     help="time the step without BGPO_FLAG_PAIR_DW (and skip the unpaired leg)")
+    ap.add_argument("--no-whole-vocab", action="store_true",
+                    help="skip the unpaired leg with the whole vocabulary as one chunk")
     ap.add_argument("--grad-variance", action="store_true",
                     help="run the Sec. 4.3 gradient std / bias vs n_t study instead")
     return ap.parse_args()
@@ -270,18 +278,22 @@ def main():
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
+        # NCCL's own start-up lines (ranks, devices) stay in the log
+        os.environ.setdefault("NCCL_DEBUG", "INFO")
+        os.environ.setdefault("NCCL_DEBUG_SUBSYS", "INIT")
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
 
     import paper_2510_11683_gb300 as bg
     from paper_2510_11683_gb300 import build as B
+    from paper_2510_11683_gb300.dp import allreduce_dw
     if not os.path.exists(B.LIB_PATH):
         B.build()
     from synth import make_inputs
 
-    # weak scaling: every rank owns B responses of a world * B batch (no collective
-    # in the data path; the dW all-reduce of an optimiser step lies outside it)
+    # weak scaling: every rank owns B responses of a world * B batch; the data
+    # path has no collective, and each step ends with the sum of dW over ranks
     wl_data, b_offset = shard_of(wl, rank, world)
     inp_cpu = make_inputs(wl_data)
     inp = {k: (v.to(dev) if v is not None else None) for k, v in inp_cpu.items()}
@@ -320,7 +332,7 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
-    def timed_leg(keep, pair_dw, ws_, sample_clocks):
+    def timed_leg(keep, pair_dw, ws_, sample_clocks, vocab_chunk=0):
         """W warm-up and K timed steps of one mode; per-kernel times from the trace."""
         def step(p):
             for j in range(n_t):
@@ -328,13 +340,16 @@ def main():
                 bg.elbo_fwd(p, j, X, W, Y, ws_, ell[j])
                 bg.bound_coeffs(p, j, ell[j], ell_old[j], A, coef[j], g[j], ws_)
                 bg.elbo_bwd_accumulate(p, j, X, W, Y, coef[j], ws_, dX, dW)
+            allreduce_dw(dW)      # the data-parallel exchange (a no-op on one rank)
 
         for _ in range(args.warmup):
-            step(bg.problem_from(wl, b_offset=b_offset, keep_logits=keep, pair_dw=pair_dw))
+            step(bg.problem_from(wl, b_offset=b_offset, keep_logits=keep, pair_dw=pair_dw,
+                                 vocab_chunk=vocab_chunk))
         torch.cuda.synchronize()
-        trace = bg.Trace(args.steps * n_t * 12 + 16)
+        chunks = -(-wl.V // (vocab_chunk or 32768))     # at most this many vocabulary chunks
+        trace = bg.Trace(args.steps * n_t * (8 + 3 * chunks) + 16)
         prob_t = bg.problem_from(wl, trace=trace, b_offset=b_offset, keep_logits=keep,
-                                 pair_dw=pair_dw)
+                                 pair_dw=pair_dw, vocab_chunk=vocab_chunk)
         clocks = ClockSampler(torch.cuda.current_device() if world == 1 else local)
         stream = torch.cuda.current_stream()
         e0 = torch.cuda.Event(enable_timing=True)
@@ -428,18 +443,25 @@ def main():
               f"{ {k: round(v[1] / args.steps, 3) for k, v in per_kernel.items()} }",
               file=sys.stderr, flush=True)
 
-    # the same step with the library's default flags (a dW GEMM per sample)
-    if rank == 0 and world == 1 and pair:
-        u_ms, u_per_kernel, _, u_launches = timed_leg(False, False, ws, False)
+    # the same step with the library's default flags (a dW GEMM per sample and
+    # vocabulary chunk, dL/dz one chunk at a time), and with the whole
+    # vocabulary as one chunk
+    legs = [("unpaired", 0)] + ([] if args.no_whole_vocab else [("unpaired_whole_vocab", 1 << 24)])
+    for leg, chunk in (legs if rank == 0 and world == 1 and pair else []):
+        ws_u = bg.alloc_workspace(bg.problem_from(wl, b_offset=b_offset, vocab_chunk=chunk), dev)
+        u_ms, u_per_kernel, _, u_launches = timed_leg(False, False, ws_u, False, chunk)
         u_roof, _, _ = rooflines(u_per_kernel, False)
-        out["unpaired"] = {
+        out[leg] = {
             "value": masked_per_step / (u_ms / 1e3), "unit": UNIT, "ms_per_step": u_ms,
-            "gpu_launches": u_launches, "roofline": u_roof,
+            "gpu_launches": u_launches, "roofline": u_roof, "vocab_chunk": chunk,
+            "workspace_bytes": ws_u.numel(),
             "per_kernel_ms_per_step": {k: v[1] / args.steps for k, v in u_per_kernel.items()}}
-        print(f"[bench] unpaired: {u_ms:.2f} ms/step, {masked_per_step / (u_ms / 1e3):.4g} tok/s, "
+        print(f"[bench] {leg}: {u_ms:.2f} ms/step, {masked_per_step / (u_ms / 1e3):.4g} tok/s, "
               f"per kernel ms/step: "
               f"{ {k: round(v[1] / args.steps, 3) for k, v in u_per_kernel.items()} }",
               file=sys.stderr, flush=True)
+        del ws_u
+        torch.cuda.empty_cache()
 
     # the same step with BGPO_FLAG_KEEP_LOGITS (the forward keeps its fp32 logits,
     # the backward forms dL/dz from them in one HBM pass instead of a fourth GEMM)
@@ -496,6 +518,7 @@ def main():
 
 def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0,
             barrier=lambda: None, pair=False):
+    from paper_2510_11683_gb300.dp import allreduce_dw
     """Same step through host buffers: every step copies its inputs (X, W, Y,
     rewards or A, l_old) from pinned host memory and reads its results (l and g)
     back. Copies run on a second stream into the other of two device buffer
@@ -548,6 +571,7 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
             bg.elbo_fwd(prob, j, b["X"], b["W"], b["Y"], ws, ell[j])
             bg.bound_coeffs(prob, j, ell[j], b["old"][j], A, coef[j], g[j], ws)
             bg.elbo_bwd_accumulate(prob, j, b["X"], b["W"], b["Y"], coef[j], ws, dX, dW)
+        allreduce_dw(dW)          # the data-parallel exchange (a no-op on one rank)
         consumed[slot].record(compute)
         out_ell.copy_(ell, non_blocking=True)
         out_g.copy_(g, non_blocking=True)

@@ -65,7 +65,7 @@
 extern "C" {
 #endif
 
-#define BGPO_ABI_VERSION 2
+#define BGPO_ABI_VERSION 3
 
 typedef enum bgpo_status {
   BGPO_OK = 0,
@@ -148,7 +148,18 @@ typedef struct bgpo_trace bgpo_trace;
  *          i >= resp_len[b] are padding and never masked (the draws of the other
  *          positions are unchanged; values outside [0, R] are clamped)
  *   flags  BGPO_FLAG_* bits (0 = defaults); other bits are rejected
- *   reserved  must be 0
+ *   vocab_chunk  columns of the vocabulary the backward handles at a time
+ *          (0 = default, else a positive multiple of 256; BGPO_ERR_INVALID_ARG
+ *          otherwise). The backward forms dL/dz, its dX contribution and its
+ *          dW rows one chunk of the vocabulary after another, so the dL/dz
+ *          buffer in the workspace holds roundup(B R, 256) x vocab_chunk
+ *          bf16 values instead of roundup(B R, 256) x V (Linearity, Sec. 3: the
+ *          gradient is a sum over vocabulary entries as well as over samples).
+ *          Default: chunks of at most 32768 columns (V split evenly, rounded
+ *          up to 256); with BGPO_FLAG_PAIR_DW, whose even samples leave their
+ *          dL/dz for the whole vocabulary pending, one chunk. A chunk of V or
+ *          more columns is the whole vocabulary at once. l and dW are the same
+ *          bits for every chunk width; dX is the same sum up to fp32 order.
  * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
  * bgpo_workspace_bytes).
  */
@@ -167,7 +178,7 @@ typedef struct bgpo_problem {
   bgpo_trace* trace;
   const int32_t* resp_len;
   uint32_t flags;
-  int32_t reserved;
+  int32_t vocab_chunk;
 } bgpo_problem;
 
 /* ABI version of the loaded library (BGPO_ABI_VERSION). */
@@ -179,15 +190,17 @@ const char* bgpo_status_string(bgpo_status status);
 /*
  * Host-only validation of a problem description (no CUDA call).
  * Returns BGPO_OK, BGPO_ERR_INVALID_ARG (NULL, bad t_mode, negative b_offset,
- * non-finite loss_scale, unknown flags, non-zero reserved) or BGPO_ERR_SHAPE.
+ * non-finite loss_scale, unknown flags, vocab_chunk negative or not a multiple
+ * of 256) or BGPO_ERR_SHAPE.
  */
 bgpo_status bgpo_validate_problem(const bgpo_problem* prob);
 
 /*
  * Bytes of device workspace the calls below need for `prob`. Depends on B, R,
- * H, V and the flags only -- never on n_t (Linearity, Sec. 3: one sample's
- * state at a time; with BGPO_FLAG_PAIR_DW two). A workspace sized with a flag
- * also serves calls made without it. Returns 0 for an invalid problem.
+ * H, V, the flags and vocab_chunk only -- never on n_t (Linearity, Sec. 3: one
+ * sample's state at a time; with BGPO_FLAG_PAIR_DW two). A workspace sized with
+ * a flag also serves calls made without it and the same vocab_chunk. Returns 0
+ * for an invalid problem.
  */
 size_t bgpo_workspace_bytes(const bgpo_problem* prob);
 
@@ -269,6 +282,15 @@ bgpo_status bgpo_vrpo_coeffs(const bgpo_problem* prob, const float* ell, const f
  *           on the tensor cores, or with BGPO_FLAG_KEEP_LOGITS read from what
  *           bgpo_elbo_fwd kept; the two give identical bits)
  *   dX[b, i, :] += W^T dz_r        dW += sum_r dz_r x_r^T
+ * computed one vocabulary chunk at a time (see bgpo_problem.vocab_chunk):
+ * dz of the chunk, then its terms of dX and of the chunk's rows of dW.
+ * Per-sample hidden states: in the paper p_theta conditions on the masked
+ * sequence (Sec. 2.1), so each MC sample may have its own X. Pass sample j's
+ * X_j to bgpo_elbo_fwd and to this call: dX then receives dL_j/dX_j, the
+ * gradient of sample j's own hidden states, added to what dX holds (zero it
+ * before each sample to read it per sample), and dW accumulates over samples.
+ * Under BGPO_FLAG_PAIR_DW the pending even sample's gathered hidden states
+ * (taken from its own X_j) stay in the workspace for the pair's dW GEMM.
  * (with BGPO_FLAG_PAIR_DW the dW term of an even sample is added by the next
  * sample's call.)
  * coef is an input (normally bgpo_bound_coeffs' output for the same j).

@@ -28,7 +28,7 @@ def _torch():
 
 
 def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=None,
-            b_offset=0, resp_len=None, keep_logits=False, pair_dw=False):
+            b_offset=0, resp_len=None, keep_logits=False, pair_dw=False, vocab_chunk=0):
     """Builds a ``bgpo_problem``; loss_scale defaults to 1/G (Algorithm 1).
 
     b_offset: global index of the first sequence (a data-parallel shard of a
@@ -40,7 +40,10 @@ def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=
     recomputing them; larger workspace, same results).
     pair_dw: sets BGPO_FLAG_PAIR_DW (samples 2k and 2k + 1 share one dW GEMM:
     dW is complete after every odd sample's backward and the last sample's,
-    not in between; larger workspace, dW equal up to fp32 summation order)."""
+    not in between; larger workspace, dW equal up to fp32 summation order).
+    vocab_chunk: columns of the vocabulary the backward handles at a time (0 =
+    the library's default; else a multiple of 256); sets the size of the
+    workspace's dL/dz buffer."""
     p = BgpoProblem()
     p.B, p.P, p.R, p.H, p.V, p.n_t, p.G, p.t_mode = B, P, R, H, V, n_t, G, t_mode
     p.seed = seed
@@ -49,16 +52,16 @@ def problem(B, P, R, H, V, n_t, G, t_mode=T_IID, seed=0, loss_scale=None, trace=
     p.resp_len = _ptr(resp_len, _torch().int32, "resp_len") if resp_len is not None else None
     p.trace = trace.handle if isinstance(trace, Trace) else trace
     p.flags = (FLAG_KEEP_LOGITS if keep_logits else 0) | (FLAG_PAIR_DW if pair_dw else 0)
-    p.reserved = 0
+    p.vocab_chunk = vocab_chunk
     return p
 
 
 def problem_from(wl, trace=None, loss_scale=None, b_offset=0, resp_len=None,
-                 keep_logits=False, pair_dw=False):
+                 keep_logits=False, pair_dw=False, vocab_chunk=0):
     """``bgpo_problem`` of a synthetic workload description (synth.Workload)."""
     return problem(wl.B, wl.P, wl.R, wl.H, wl.V, wl.n_t, wl.G, wl.t_mode, wl.seed,
                    loss_scale=loss_scale, trace=trace, b_offset=b_offset, resp_len=resp_len,
-                   keep_logits=keep_logits, pair_dw=pair_dw)
+                   keep_logits=keep_logits, pair_dw=pair_dw, vocab_chunk=vocab_chunk)
 
 
 def validate_problem(prob):

@@ -23,7 +23,7 @@ class BgpoProblem(ctypes.Structure):
         ("n_t", c_int32), ("G", c_int32), ("t_mode", c_int32),
         ("seed", ctypes.c_uint64), ("loss_scale", ctypes.c_float), ("b_offset", c_int32),
         ("trace", c_void_p), ("resp_len", c_void_p),
-        ("flags", ctypes.c_uint32), ("reserved", c_int32),
+        ("flags", ctypes.c_uint32), ("vocab_chunk", c_int32),
     ]
 
 

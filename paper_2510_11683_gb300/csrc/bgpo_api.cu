@@ -65,8 +65,8 @@ bgpo_status check_problem(const bgpo_problem* p) {
   if (p->t_mode != BGPO_T_IID && p->t_mode != BGPO_T_STRATIFIED) return BGPO_ERR_INVALID_ARG;
   if (p->b_offset < 0) return BGPO_ERR_INVALID_ARG;
   if (!isfinite(p->loss_scale)) return BGPO_ERR_INVALID_ARG;
-  if ((p->flags & ~(BGPO_FLAG_KEEP_LOGITS | BGPO_FLAG_PAIR_DW)) != 0u || p->reserved != 0)
-    return BGPO_ERR_INVALID_ARG;
+  if ((p->flags & ~(BGPO_FLAG_KEEP_LOGITS | BGPO_FLAG_PAIR_DW)) != 0u) return BGPO_ERR_INVALID_ARG;
+  if (p->vocab_chunk < 0 || p->vocab_chunk % kBN != 0) return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
   if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
@@ -76,11 +76,13 @@ bgpo_status check_problem(const bgpo_problem* p) {
   return BGPO_OK;
 }
 
-Geometry geometry_of(const bgpo_problem* p) { return make_geometry(p->B, p->P, p->R, p->H, p->V); }
-
 bool keeps_logits(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_KEEP_LOGITS) != 0u; }
 
 bool pairs_dw(const bgpo_problem* p) { return (p->flags & BGPO_FLAG_PAIR_DW) != 0u; }
+
+Geometry geometry_of(const bgpo_problem* p) {
+  return make_geometry(p->B, p->P, p->R, p->H, p->V, p->vocab_chunk, pairs_dw(p));
+}
 
 bgpo_status check_sample(const bgpo_problem* p, int32_t j) {
   return (j >= 0 && j < p->n_t) ? BGPO_OK : BGPO_ERR_INVALID_ARG;
@@ -331,17 +333,18 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   const bool pair = pairs_dw(prob);
   const bool defer = pair && j % 2 == 0 && j + 1 < prob->n_t;
   const uint64_t zr = (uint64_t)w.dz_rows;
+  const uint64_t zc = (uint64_t)w.dz_cols;
   CUtensorMap map_xm_k, map_w_k, map_dz_k, map_w_mn, map_dz_mn, map_xmT_k;
   CUtensorMap map_dz_st, map_dxp_st, map_dw_red;
   const uint64_t dxp_rows = (uint64_t)dxp_row_block_cap(g) * kPairM;
   if (!map_2d(&map_xm_k, w.xm, g.H, g.m_pad, g.H * 2, kBK, kBM) ||
       !map_2d(&map_w_k, W, g.H, g.V, g.H * 2, kBK, kBNHalf) ||
-      !map_2d(&map_dz_k, w.dz, g.v_pad, zr, g.v_pad * 2, kBK, kBM) ||
+      !map_2d(&map_dz_k, w.dz, zc, zr, zc * 2, kBK, kBM) ||
       !map_2d(&map_w_mn, W, g.H, g.V, g.H * 2, 64, kBK) ||
-      !map_2d(&map_dz_mn, w.dz, g.v_pad, zr, g.v_pad * 2, 64, kBK) ||
+      !map_2d(&map_dz_mn, w.dz, zc, zr, zc * 2, 64, kBK) ||
       !map_2d(&map_xmT_k, w.xmT, zr, g.H, zr * 2, kBK, kBNHalf) ||
       // epilogue destinations: 32-row sub-tiles of 128 bytes
-      !map_2d(&map_dz_st, w.dz, g.v_pad, zr, g.v_pad * 2, 64, 32) ||
+      !map_2d(&map_dz_st, w.dz, zc, zr, zc * 2, 64, 32) ||
       !map_2d(&map_dxp_st, w.dxp, g.H, dxp_rows, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32) ||
       !map_2d(&map_dw_red, dW, g.H, g.V, g.H * 4, 32, 32, CU_TENSOR_MAP_DATA_TYPE_FLOAT32))
     return BGPO_ERR_CUDA;
@@ -353,28 +356,47 @@ bgpo_status bgpo_elbo_bwd_accumulate(const bgpo_problem* prob, int32_t j, const 
   ga.dW = dW;
   ga.dX = dX;
   ga.pair_consume = pair && (j & 1);
-  if (keep) {
-    TraceScope ts(prob->trace, KID_DZ_FROM_LOGITS, s);
-    if (launch_dz_from_logits(g, j, coef, sms, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
-  } else {
-    TraceScope ts(prob->trace, KID_LMHEAD_DZ, s);
-    if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, map_dz_st, ga, w, s) != cudaSuccess)
-      return BGPO_ERR_CUDA;
-  }
   {
-    TraceScope ts(prob->trace, KID_DX_GEMM, s);
-    if (launch_gemm(GEMM_DX, map_dz_k, map_w_mn, map_dxp_st, ga, w, s) != cudaSuccess)
-      return BGPO_ERR_CUDA;
+    // Xm^T for the dW GEMMs; also records the dW pairing state of this sample
+    TraceScope ts(prob->trace, KID_XM_TRANSPOSE, s);
+    if (launch_xm_transpose(g, j, defer, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+  }
+  // One vocabulary chunk at a time (Linearity, Sec. 3, within a sample: the
+  // gradient is a sum over vocabulary entries too): dZ of the chunk, its dX
+  // contribution, and, when dZ holds one chunk, the chunk's rows of dW.
+  for (int64_t c = 0; c < g.n_vc; ++c) {
+    ga.v_begin = chunk_begin(g, c);
+    ga.v_end = chunk_end(g, c);
+    ga.dz_col0 = w.dz_chunk_local ? 0 : ga.v_begin;
+    ga.chunk = c;
+    if (keep) {
+      TraceScope ts(prob->trace, KID_DZ_FROM_LOGITS, s);
+      if (launch_dz_from_logits(g, j, c, coef, sms, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
+    } else {
+      TraceScope ts(prob->trace, KID_LMHEAD_DZ, s);
+      if (launch_gemm(GEMM_DZ, map_xm_k, map_w_k, map_dz_st, ga, w, s) != cudaSuccess)
+        return BGPO_ERR_CUDA;
+    }
+    {
+      TraceScope ts(prob->trace, KID_DX_GEMM, s);
+      if (launch_gemm(GEMM_DX, map_dz_k, map_w_mn, map_dxp_st, ga, w, s) != cudaSuccess)
+        return BGPO_ERR_CUDA;
+    }
+    if (w.dz_chunk_local) {
+      TraceScope ts(prob->trace, KID_DW_GEMM, s);
+      if (launch_gemm(GEMM_DW, map_dz_mn, map_xmT_k, map_dw_red, ga, w, s) != cudaSuccess)
+        return BGPO_ERR_CUDA;
+    }
   }
   {
     TraceScope ts(prob->trace, KID_DX_REDUCE, s);
     if (launch_dx_reduce(g, j, w, dX, s) != cudaSuccess) return BGPO_ERR_CUDA;
   }
-  {
-    TraceScope ts(prob->trace, KID_XM_TRANSPOSE, s);
-    if (launch_xm_transpose(g, j, defer, w, s) != cudaSuccess) return BGPO_ERR_CUDA;
-  }
-  if (!defer) {
+  if (!w.dz_chunk_local && !defer) {
+    // dZ spans the whole vocabulary (one chunk, or dW pairing): one dW GEMM
+    ga.v_begin = 0;
+    ga.v_end = g.V;
+    ga.dz_col0 = 0;
     TraceScope ts(prob->trace, KID_DW_GEMM, s);
     if (launch_gemm(GEMM_DW, map_dz_mn, map_xmT_k, map_dw_red, ga, w, s) != cudaSuccess)
       return BGPO_ERR_CUDA;

@@ -23,8 +23,10 @@ struct WsPtrs {
   float2* part;
   void* xm;   // bf16
   void* xmT;  // bf16 [H, dz_rows]
-  void* dz;   // bf16 [dz_rows, v_pad]
+  void* dz;   // bf16 [dz_rows, dz_cols]
   int64_t dz_rows;
+  int64_t dz_cols;     // vc (one vocabulary chunk at a time) or v_pad (the whole vocabulary)
+  bool dz_chunk_local; // chunk c of dZ starts at column 0 (else at column c vc)
   float* dxp;
   float* zc;  // fp32 logits kept by the forward; null when the layout has none
 };
@@ -49,9 +51,10 @@ cudaError_t launch_gather(const Geometry& g, int32_t j, const void* X, const int
 // `kept_logits`: the forward GEMM just wrote this sample's logits to w.zc.
 cudaError_t launch_lse_combine(const Geometry& g, int32_t j, bool kept_logits, const WsPtrs& w,
                                cudaStream_t s);
-// dz from the logits the forward kept (same arithmetic as the GEMM_DZ epilogue).
-cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, const float* coef, int num_sms,
-                                  const WsPtrs& w, cudaStream_t s);
+// dz of vocabulary chunk `chunk` from the logits the forward kept (same
+// arithmetic as the GEMM_DZ epilogue).
+cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, int64_t chunk, const float* coef,
+                                  int num_sms, const WsPtrs& w, cudaStream_t s);
 cudaError_t launch_seq_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* ell_out,
                               cudaStream_t s);
 cudaError_t launch_bound_coeffs(int32_t B, int32_t n_t, float loss_scale, const float* ell,
@@ -78,6 +81,11 @@ struct GemmArgs {
   Geometry g;
   int num_pairs;      // CTA pairs launched (gemm_num_pairs)
   int32_t j;
+  // GEMM_DZ / GEMM_DX / GEMM_DW: the vocabulary range [v_begin, v_end) of this
+  // launch (one chunk of the backward, or the whole vocabulary for a dW GEMM
+  // over a whole-vocabulary dZ) and the dZ column where v_begin lies
+  int64_t v_begin = 0, v_end = 0, dz_col0 = 0;
+  int64_t chunk = 0;  // GEMM_DX: chunk index (chunk 0 stores split partials, later ones add)
   const float* coef;  // GEMM_DZ: per-sequence dL/dl
   float* dW;          // GEMM_DW: accumulated weight gradient [V, H]
   float* dX = nullptr;  // GEMM_DX: accumulated dHidden [B, R, H] (written directly without split-K)

@@ -25,6 +25,10 @@ constexpr int kBK = 64;          // K per pipeline stage: one 128-byte swizzle r
 constexpr int kUmmaK = 16;       // K of one tcgen05.mma kind::f16 instruction
 constexpr int kStages = 6;       // TMA -> MMA pipeline depth
 constexpr int kMaxSplits = 16;   // split-K limit of the dX GEMM
+// Widest vocabulary chunk of the backward by default: dZ is formed, used by
+// the dX GEMM and the dW GEMM one chunk of at most this many columns at a
+// time, so its buffer holds M x V_c instead of M x V.
+constexpr int64_t kVChunkDefault = 32768;
 
 constexpr uint32_t kTileABytes = kBM * kBK * 2;       // 16 KB per CTA
 constexpr uint32_t kTileBBytes = kBNHalf * kBK * 2;   // 16 KB per CTA
@@ -81,18 +85,40 @@ BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_pairs, int64_t k_bloc
   return best;
 }
 
+// Width of the backward's vocabulary chunks. `request` 0 asks for the
+// default: one chunk when dW pairing keeps the whole vocabulary's dZ anyway,
+// else the V columns split into ceil(V / kVChunkDefault) chunks of equal
+// width rounded up to a tile. A positive request is a multiple of kBN (the
+// host validates it). A width of V or more is a single chunk.
+BGPO_HD int64_t vocab_chunk_width(int64_t V, int64_t request, bool pair_dw) {
+  int64_t w;
+  if (request > 0) {
+    w = request;
+  } else if (pair_dw) {
+    w = V;
+  } else {
+    const int64_t n = ceil_div(V, kVChunkDefault);
+    w = round_up(ceil_div(V, n), kBN);
+  }
+  return w >= V ? round_up(V, 64) : w;
+}
+
 // Geometry derived from the problem sizes (host and device agree on it).
 struct Geometry {
   int64_t B, P, R, H, V;
   int64_t m_cap;      // B * R: most masked rows a sample can have
   int64_t m_pad;      // m_cap rounded up to a pair tile of rows
-  int64_t v_pad;      // V rounded up to 64 (row pitch of the dZ buffer)
+  int64_t v_pad;      // V rounded up to 64 (row pitch of the kept logits)
   int64_t n_vt;       // vocabulary tiles of kBN columns
   int64_t tiles_h;    // hidden-size tiles of kBN columns
-  int64_t kb_v;       // K blocks of kBK over the vocabulary (dX GEMM)
+  int64_t kb_v;       // K blocks of kBK over the vocabulary
+  int64_t vc;         // vocabulary chunk width of the backward (v_pad when one chunk)
+  int64_t n_vc;       // vocabulary chunks: chunk c covers [c vc, min(V, (c + 1) vc))
+  int64_t kb_vc_min;  // K blocks of kBK of the narrowest chunk (the dX split bound)
 };
 
-BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64_t V) {
+BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64_t V,
+                               int64_t vchunk_request = 0, bool pair_dw = false) {
   Geometry g;
   g.B = B; g.P = P; g.R = R; g.H = H; g.V = V;
   g.m_cap = B * R;
@@ -101,7 +127,18 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
   g.n_vt = ceil_div(V, kBN);
   g.tiles_h = ceil_div(H, kBN);
   g.kb_v = ceil_div(V, kBK);
+  g.vc = vocab_chunk_width(V, vchunk_request, pair_dw);
+  g.n_vc = ceil_div(V, g.vc);
+  const int64_t last = V - (g.n_vc - 1) * g.vc;
+  g.kb_vc_min = ceil_div(last < g.vc ? last : g.vc, kBK);
   return g;
+}
+
+// Vocabulary range [v0, v1) of backward chunk c.
+BGPO_HD int64_t chunk_begin(const Geometry& g, int64_t c) { return c * g.vc; }
+BGPO_HD int64_t chunk_end(const Geometry& g, int64_t c) {
+  const int64_t e = (c + 1) * g.vc;
+  return e < g.V ? e : g.V;
 }
 
 // Device workspace layout. Every region starts on a 1024-byte boundary (TMA
@@ -121,8 +158,11 @@ struct WsLayout {
   size_t fwd_bytes;  // end of the regions a forward pass uses (err .. xm); the same under
                      // every flag
   size_t xmT;        // bf16[H * dz_rows] the same, transposed (the dW GEMM's K-major operand)
-  size_t dz;         // bf16[dz_rows * v_pad] dL/dz of the current sample (and of a pending one)
+  size_t dz;         // bf16[dz_rows * dz_cols] dL/dz of the current sample (and of a pending
+                     // one): one vocabulary chunk at a time, or the whole vocabulary
   size_t dz_rows;    // m_pad, or 2 m_pad when the dW GEMM pairs samples
+  size_t dz_cols;    // vc when the buffer holds one chunk, v_pad when it holds them all
+  bool dz_chunk_local;  // chunk c is formed at column 0 (else at column c vc)
   size_t dxp;        // float[dxp_elems] split-K partials of dX
   size_t dxp_elems;
   size_t zc;         // float[m_pad * v_pad] logits kept by the forward (last region)
@@ -145,11 +185,14 @@ BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
 
 // `keep_logits` appends the fp32 logit region. `pair_dw` doubles the rows of
 // dZ and the columns of Xm^T: the rows of an even sample wait there for the
-// dW GEMM of the next sample, whose rows follow them.
+// dW GEMM of the next sample, whose rows follow them; its dZ rows then span
+// the whole vocabulary. Otherwise dZ holds one vocabulary chunk.
 BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits, bool pair_dw) {
   WsLayout L;
   size_t o = 0;
   L.dz_rows = (pair_dw ? 2 : 1) * (size_t)g.m_pad;
+  L.dz_chunk_local = !pair_dw && g.n_vc > 1;
+  L.dz_cols = L.dz_chunk_local ? (size_t)g.vc : (size_t)g.v_pad;
   L.err = o;       o = align_ws(o + 64);
   L.t = o;         o = align_ws(o + 4 * (size_t)g.B);
   L.tnum = o;      o = align_ws(o + 8 * (size_t)g.B);
@@ -163,7 +206,7 @@ BGPO_HD WsLayout make_ws_layout(const Geometry& g, bool keep_logits, bool pair_d
   L.xm = o;        o = align_ws(o + 2 * (size_t)g.m_pad * (size_t)g.H);
   L.fwd_bytes = o;
   L.xmT = o;       o = align_ws(o + 2 * (size_t)g.H * L.dz_rows);
-  L.dz = o;        o = align_ws(o + 2 * L.dz_rows * (size_t)g.v_pad);
+  L.dz = o;        o = align_ws(o + 2 * L.dz_rows * L.dz_cols);
   L.dxp_elems = (size_t)dxp_row_block_cap(g) * kPairM * (size_t)g.H;
   L.dxp = o;       o = align_ws(o + 4 * L.dxp_elems);
   L.zc_bytes = keep_logits ? 4 * (size_t)g.m_pad * (size_t)g.v_pad : 0;

@@ -21,14 +21,17 @@
 //             and the target logit (Eq. 4: log softmax gathered at y^i); when
 //             the workspace has a logit region the fp32 tile also leaves
 //             through TMA stores, for the backward.
-//   GEMM_DZ   z = Xm W^T recomputed (when the forward kept no logits);
-//             epilogue: dz = w_r (onehot - e^{z - lse}) stored as bf16
-//             (gradient of Eq. 4 weighted by Eq. 13's dL/dl).
-//   GEMM_DX   dXm = dZ W (K = vocabulary): split-K partials in fp32, or, when
-//             the launch needs no split, added straight into the dX rows.
-//   GEMM_DW   dW += dZ^T Xm (K = masked rows; Xm read as its transpose, so
-//             that the B operand is K-major), fp32 TMA reduce-add. With dW
-//             pairing, K also covers the rows of the pending sample before.
+//   GEMM_DZ   z = Xm W^T recomputed (when the forward kept no logits) for one
+//             vocabulary chunk of the backward; epilogue: dz = w_r (onehot -
+//             e^{z - lse}) stored as bf16 (gradient of Eq. 4 weighted by
+//             Eq. 13's dL/dl).
+//   GEMM_DX   dXm += dZ_c W_c (K = the chunk's vocabulary): split-K partials in
+//             fp32, stored by the first chunk and added by the later ones, or,
+//             when the launch needs no split, added straight into the dX rows.
+//   GEMM_DW   dW[chunk rows] += dZ_c^T Xm (K = masked rows; Xm read as its
+//             transpose, so that the B operand is K-major), fp32 TMA
+//             reduce-add. With dW pairing (whole-vocabulary dZ), K also covers
+//             the rows of the pending sample before.
 //
 // Every wait is bounded (time and polls); a wait that runs out sets the
 // workspace error word to BGPO_ERR_TIMEOUT and both CTAs drain and exit.
@@ -55,6 +58,7 @@ struct GemmParams {
   Geometry g;
   int num_pairs;
   int32_t j;
+  int64_t v_begin, v_end, dz_col0, chunk;
   WsPtrs w;
   const float* coef;
   float* dW;
@@ -83,19 +87,21 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_
   w.kb_first = 0;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
     w.tiles_m = ceil_div(M, kPairM);
-    w.tiles_n = p.g.n_vt;
+    w.tiles_n = KIND == GEMM_FWD ? p.g.n_vt : ceil_div(p.v_end - p.v_begin, kBN);
     w.kb_total = p.g.H / kBK;
     w.units = w.tiles_m * w.tiles_n;
   } else if (KIND == GEMM_DX) {
     w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = p.g.tiles_h;
-    w.kb_total = p.g.kb_v;
-    w.splits = w.tiles_m > 0 ? dx_splits(w.tiles_m, w.tiles_n, p.num_pairs, w.kb_total,
+    w.kb_total = ceil_div(p.v_end - p.v_begin, kBK);
+    // one split count for every chunk of the sample (the partials of split s
+    // accumulate over the chunks), bounded by the narrowest chunk's K blocks
+    w.splits = w.tiles_m > 0 ? dx_splits(w.tiles_m, w.tiles_n, p.num_pairs, p.g.kb_vc_min,
                                          dxp_row_block_cap(p.g))
                              : 1;
     w.units = w.tiles_m * w.tiles_n * w.splits;
   } else {  // GEMM_DW
-    w.tiles_m = ceil_div(p.g.V, kPairM);
+    w.tiles_m = ceil_div(p.v_end - p.v_begin, kPairM);
     w.tiles_n = p.g.tiles_h;
     w.kb_total = ceil_div(roff + M, kBK);
     w.kb_first = k0 / kBK;
@@ -162,18 +168,26 @@ __device__ __forceinline__ int64_t b_rows(const GemmParams& p) {
   return KIND == GEMM_DW ? p.g.H : p.g.V;
 }
 
+// First row of the K-major B operand in this launch: dZ's W rows start at the
+// chunk's first vocabulary entry.
+template <int KIND>
+__device__ __forceinline__ int64_t b_base(const GemmParams& p) {
+  return KIND == GEMM_DZ ? p.v_begin : 0;
+}
+
 // Bytes this CTA's copies deliver for one stage of unit t (boxes that would lie
 // wholly outside the operand are not issued; their MMA outputs are discarded).
 template <int KIND>
 __device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit& t, uint32_t rank) {
-  const int32_t a0 = t.m_blk * kPairM + (int32_t)rank * kBM;
-  const int32_t b0 = t.n_blk * kBN + (int32_t)rank * kBNHalf;
+  const int64_t a0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM;
+  const int64_t b0 = b_base<KIND>(p) + (int64_t)t.n_blk * kBN + (int64_t)rank * kBNHalf;
   uint32_t bytes = 0;
   if (!Majors<KIND>::a_mn) {
     bytes += kTileABytes;
   } else {
+    // dZ^T vocabulary columns of this CTA inside the dZ buffer
     for (int c = 0; c < kBM / 64; ++c)
-      if (a0 + c * 64 < p.g.v_pad) bytes += kMnChunkBytes;
+      if (p.dz_col0 + a0 + c * 64 < p.w.dz_cols) bytes += kMnChunkBytes;
   }
   if (!Majors<KIND>::b_mn) {
     if (b0 < b_rows<KIND>(p)) bytes += kTileBBytes;
@@ -186,7 +200,8 @@ __device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit&
 
 // Issues this CTA's TMA loads of one stage; they complete on `cbar`, the even
 // CTA's full barrier (shared::cluster address). The dX GEMM's dZ rows start at
-// `roff`.
+// `roff`; its K blocks count from the chunk's first vocabulary entry, which
+// lies at dZ column dz_col0 and W row v_begin.
 template <int KIND>
 __device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMap* ma,
                                            const CUtensorMap* mb, uint32_t sa, uint32_t sb,
@@ -194,24 +209,28 @@ __device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMa
                                            uint32_t rank, int64_t roff) {
   const int32_t a0 =
       t.m_blk * kPairM + (int32_t)rank * kBM + (KIND == GEMM_DX ? (int32_t)roff : 0);
-  const int32_t b0 = t.n_blk * kBN + (int32_t)rank * kBNHalf;
+  const int64_t b0 = b_base<KIND>(p) + (int64_t)t.n_blk * kBN + (int64_t)rank * kBNHalf;
   if (!Majors<KIND>::a_mn) {
-    tma_load_2d_pair(sa, ma, cbar, kb * kBK, a0);
+    const int32_t ka = kb * kBK + (KIND == GEMM_DX ? (int32_t)p.dz_col0 : 0);
+    tma_load_2d_pair(sa, ma, cbar, ka, a0);
   } else {
     // dZ^T rows of this CTA: 2 boxes of 64 vocabulary columns x 64 masked rows
 #pragma unroll
-    for (int c = 0; c < kBM / 64; ++c)
-      if (a0 + c * 64 < p.g.v_pad)
-        tma_load_2d_pair(sa + c * kMnChunkBytes, ma, cbar, a0 + c * 64, kb * kBK);
+    for (int c = 0; c < kBM / 64; ++c) {
+      const int64_t xa = p.dz_col0 + a0 + c * 64;
+      if (xa < p.w.dz_cols)
+        tma_load_2d_pair(sa + c * kMnChunkBytes, ma, cbar, (int32_t)xa, kb * kBK);
+    }
   }
   if (!Majors<KIND>::b_mn) {
-    if (b0 < b_rows<KIND>(p)) tma_load_2d_pair(sb, mb, cbar, kb * kBK, b0);
+    if (b0 < b_rows<KIND>(p)) tma_load_2d_pair(sb, mb, cbar, kb * kBK, (int32_t)b0);
   } else {
-    // W columns of this CTA (GEMM_DX): 2 boxes of 64 x 64
+    // W columns of this CTA (GEMM_DX): 2 boxes of 64 x 64, rows from the chunk's start
+    const int32_t kw = (int32_t)(p.v_begin + (int64_t)kb * kBK);
 #pragma unroll
     for (int c = 0; c < kBNHalf / 64; ++c)
       if (b0 + c * 64 < p.g.H)
-        tma_load_2d_pair(sb + c * kMnChunkBytes, mb, cbar, b0 + c * 64, kb * kBK);
+        tma_load_2d_pair(sb + c * kMnChunkBytes, mb, cbar, (int32_t)b0 + c * 64, kw);
   }
 }
 
@@ -317,7 +336,8 @@ __device__ __forceinline__ void epi_fwd(const GemmParams& p, const CUtensorMap* 
 
 // GEMM_DZ: dz_{r,v} = w_r (1[v = y_r] - e^{z_{r,v} - lse_r}) as bf16, zero for
 // rows >= M and vocabulary columns >= V; 64-column sub-tiles leave through TMA
-// stores into dZ [dz_rows, v_pad], from row `roff` on.
+// stores into dZ [dz_rows, dz_cols], from row `roff` on; vocabulary entry v
+// lands in column v - v_begin + dz_col0.
 __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
                                        const Unit& t, int64_t row0, int64_t roff, int lane,
                                        uint32_t tb, EpiStage& st) {
@@ -332,12 +352,13 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
     lse_l2 = p.w.lse[r] * kLog2e;
     y = p.w.tgt[r];
   }
-  const int32_t v0 = t.n_blk * kBN;
+  const int32_t v0 = (int32_t)p.v_begin + t.n_blk * kBN;
   const int32_t V = (int32_t)p.g.V;
+  const int32_t shift = (int32_t)(p.dz_col0 - p.v_begin);   // vocabulary entry -> dZ column
 #pragma unroll 1
   for (int c = 0; c < kBN / 64; ++c) {
     const int32_t col0 = v0 + c * 64;
-    if (col0 >= p.g.v_pad) break;  // warp-uniform
+    if (col0 + shift >= p.w.dz_cols) break;  // warp-uniform
     uint4 chunk[8];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -365,16 +386,18 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
     const uint32_t sbuf = st.acquire(lane);
     stage_row(sbuf, lane, chunk);
     st.release(lane, sbuf,
-               [&](uint32_t a) { tma_store_2d(map_c, a, col0, (int32_t)(row0 + roff)); });
+               [&](uint32_t a) { tma_store_2d(map_c, a, col0 + shift, (int32_t)(row0 + roff)); });
   }
 }
 
 // GEMM_DX: fp32 partial of split s, rows [split * tiles_m * 256 + r] of the
-// partial buffer, 32-column sub-tiles through TMA stores (rows >= M hold zeros).
-// Without split-K every dX element has exactly this one contribution in the
-// launch, so the lane adds its row's sub-tile straight into dX[b, i] (the row
-// the compaction recorded), 128 contiguous bytes per sub-tile, and the split
-// reduction after the GEMM has nothing to do.
+// partial buffer, 32-column sub-tiles through TMA stores in the first
+// vocabulary chunk and TMA reduce-adds in the later ones (every element has one
+// writer per launch and the chunks run in order, so the sum is deterministic;
+// rows >= M hold zeros). Without split-K every dX element has exactly this one
+// contribution in the launch, so the lane adds its row's sub-tile straight
+// into dX[b, i] (the row the compaction recorded), 128 contiguous bytes per
+// sub-tile, and the split reduction after the last chunk has nothing to do.
 __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
                                        const Work& wk, const Unit& t, int64_t row0, int lane,
                                        uint32_t tb, EpiStage& st) {
@@ -411,16 +434,22 @@ __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* m
       chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
     const uint32_t sbuf = st.acquire(lane);
     stage_row(sbuf, lane, chunk);
-    st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, h0 + c * 32, prow0); });
+    if (p.chunk == 0)
+      st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, h0 + c * 32, prow0); });
+    else
+      st.release(lane, sbuf,
+                 [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, prow0); });
   }
 }
 
 // GEMM_DW: dW[v, h] += acc through TMA reduce-add of 32 x 32 fp32 sub-tiles
 // (the read-modify-write happens at L2; vocabulary rows >= V are clipped).
+// Accumulator row r is vocabulary entry v_begin + r.
 __device__ __forceinline__ void epi_dw(const GemmParams& p, const CUtensorMap* map_c, const Unit& t,
                                        int64_t row0, int lane, uint32_t tb, EpiStage& st) {
   const int32_t h0 = t.n_blk * kBN;
-  if (row0 >= p.g.V) return;  // this warp's rows all lie past the vocabulary (warp-uniform)
+  const int64_t v = p.v_begin + row0;
+  if (v >= p.g.V) return;  // this warp's rows all lie past the vocabulary (warp-uniform)
 #pragma unroll 1
   for (int c = 0; c < kBN / 32; ++c) {
     if (h0 + c * 32 >= p.g.H) break;  // warp-uniform
@@ -434,7 +463,7 @@ __device__ __forceinline__ void epi_dw(const GemmParams& p, const CUtensorMap* m
     const uint32_t sbuf = st.acquire(lane);
     stage_row(sbuf, lane, chunk);
     st.release(lane, sbuf,
-               [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, (int32_t)row0); });
+               [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, (int32_t)v); });
   }
 }
 
@@ -700,6 +729,10 @@ cudaError_t launch_gemm(GemmKind kind, const CUtensorMap& map_a, const CUtensorM
   p.g = a.g;
   p.num_pairs = a.num_pairs;
   p.j = a.j;
+  p.v_begin = a.v_begin;
+  p.v_end = a.v_end;
+  p.dz_col0 = a.dz_col0;
+  p.chunk = a.chunk;
   p.w = w;
   p.coef = a.coef;
   p.dW = a.dW;

@@ -238,14 +238,16 @@ __global__ void __launch_bounds__(256) k_lse_combine(Geometry g, int32_t j, bool
 }
 
 // ---------------------------------------------------------------------------
-// dL/dz of the masked rows from the logits the forward kept:
+// dL/dz of the masked rows, one vocabulary chunk [v0, v1) of the backward, from
+// the logits the forward kept:
 //   dz_{r,v} = w_r (1[v = y_r] - e^{z_{r,v} - lse_r}),  w_r = coef_b / t_b
 // (gradient of Eq. 4 weighted by dL/dl), bf16, zero for rows in
-// [M, round_up(M, 256)) and columns in [V, v_pad): the arithmetic of the
+// [M, round_up(M, 256)) and columns at or past V: the arithmetic of the
 // GEMM_DZ epilogue on the same fp32 logits, so both give identical bits.
-// HBM-bound: each row streams 4 v_pad bytes in and 2 v_pad bytes out. Work
-// items are (row, 8192-column chunk); each thread has kDzVec independent
-// 32-byte loads in flight before it computes.
+// Entry v lands in dZ column v - v0 (a chunk-local buffer) or v (a
+// whole-vocabulary one). HBM-bound: each row streams 4 bytes in and 2 bytes out
+// per column. Work items are (row, 8192-column piece); each thread has kDzVec
+// independent 32-byte loads in flight before it computes.
 // When the workspace holds no logits of sample j the kernel records
 // BGPO_ERR_INVALID_ARG and invalidates the sample tag, so that the dX / dW
 // kernels after it do no work.
@@ -255,7 +257,8 @@ constexpr int kDzVec = 4;                           // 8-column vectors per thre
 constexpr int kDzItemVecs = kDzThreads * kDzVec;    // 1024 vectors = 8192 columns
 
 __global__ void __launch_bounds__(kDzThreads, 4)
-    k_dz_from_logits(Geometry g, int32_t j, const float* __restrict__ coef, WsPtrs w) {
+    k_dz_from_logits(Geometry g, int32_t j, int64_t chunk, const float* __restrict__ coef,
+                     WsPtrs w) {
   const int32_t M = rows_of_sample(w.err, j, KID_DZ_FROM_LOGITS);
   if (w.err[ERR_LOGITS] != 1) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -265,13 +268,19 @@ __global__ void __launch_bounds__(kDzThreads, 4)
     return;
   }
   if (!BGPO_IN_BOUNDS(w.err, M <= g.m_cap, KID_DZ_FROM_LOGITS * 16 + 9)) return;
-  const int64_t nvec = g.v_pad / 8;
+  const int64_t v_begin = chunk_begin(g, chunk);
+  // 8-column vectors of the chunk (its width rounded up to 64 columns), of a
+  // kept-logit row and of a dZ row
+  const int64_t nvec = round_up(chunk_end(g, chunk) - v_begin, 64) / 8;
+  const int64_t zvec = g.v_pad / 8;
+  const int64_t dvec = w.dz_cols / 8;
   const int64_t per_row = ceil_div(nvec, kDzItemVecs);
   const int64_t items = round_up(M, kPairM) * per_row;
-  const float4* __restrict__ zc = reinterpret_cast<const float4*>(w.zc);
+  const float4* __restrict__ zc = reinterpret_cast<const float4*>(w.zc) + v_begin / 4;
   // this sample's dZ rows start at the pairing offset (0 without pairing)
   uint4* __restrict__ dz = reinterpret_cast<uint4*>(w.dz) +
-                           row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad) * nvec;
+                           row_offset(w.err[ERR_ROW_OFF], w.dz_rows, g.m_pad) * dvec +
+                           (w.dz_chunk_local ? 0 : v_begin / 8);
   const int32_t V = (int32_t)g.V;
   for (int64_t q = blockIdx.x; q < items; q += gridDim.x) {
     const int64_t r = q / per_row;
@@ -292,7 +301,7 @@ __global__ void __launch_bounds__(kDzThreads, 4)
     for (int k = 0; k < kDzVec; ++k) {
       const int64_t v = v0 + k * kDzThreads;
       if (valid && v < nvec) {
-        const float4* src = zc + (r * nvec + v) * 2;
+        const float4* src = zc + r * zvec * 2 + v * 2;
         z[k][0] = __ldcs(src);
         z[k][1] = __ldcs(src + 1);
       } else {
@@ -311,7 +320,7 @@ __global__ void __launch_bounds__(kDzThreads, 4)
         float d[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const int32_t col = (int32_t)(v * 8) + e + h;
+          const int32_t col = (int32_t)(v_begin + v * 8) + e + h;
           const float pr = exp2f(fmaf(zz[e + h], kLog2e, -lse_l2));
           const float val = wr * ((col == y ? 1.f : 0.f) - pr);
           d[h] = (valid && col < V) ? val : 0.f;
@@ -319,7 +328,7 @@ __global__ void __launch_bounds__(kDzThreads, 4)
         const __nv_bfloat162 hv = __floats2bfloat162_rn(d[0], d[1]);
         packed[e / 2] = *reinterpret_cast<const uint32_t*>(&hv);
       }
-      dz[r * nvec + v] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+      dz[r * dvec + v] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
     }
   }
 }
@@ -549,6 +558,8 @@ WsPtrs ws_pointers(void* ws, const WsLayout& L, bool forward_only) {
   p.xmT = forward_only ? nullptr : base + L.xmT;
   p.dz = forward_only ? nullptr : base + L.dz;
   p.dz_rows = forward_only ? 0 : (int64_t)L.dz_rows;
+  p.dz_cols = forward_only ? 0 : (int64_t)L.dz_cols;
+  p.dz_chunk_local = !forward_only && L.dz_chunk_local;
   p.dxp = forward_only ? nullptr : reinterpret_cast<float*>(base + L.dxp);
   p.zc = (!forward_only && L.zc_bytes) ? reinterpret_cast<float*>(base + L.zc) : nullptr;
   return p;
@@ -573,12 +584,12 @@ cudaError_t launch_lse_combine(const Geometry& g, int32_t j, bool kept_logits, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, const float* coef, int num_sms,
-                                  const WsPtrs& w, cudaStream_t s) {
+cudaError_t launch_dz_from_logits(const Geometry& g, int32_t j, int64_t chunk, const float* coef,
+                                  int num_sms, const WsPtrs& w, cudaStream_t s) {
   // 4 resident CTAs per SM; never more CTAs than the largest sample has items
-  const int64_t most = g.m_pad * ceil_div(g.v_pad / 8, kDzItemVecs);
+  const int64_t most = g.m_pad * ceil_div(g.vc / 8, kDzItemVecs);
   const int64_t grid = most < 4 * (int64_t)num_sms ? most : 4 * (int64_t)num_sms;
-  k_dz_from_logits<<<(unsigned)grid, kDzThreads, 0, s>>>(g, j, coef, w);
+  k_dz_from_logits<<<(unsigned)grid, kDzThreads, 0, s>>>(g, j, chunk, coef, w);
   return cudaGetLastError();
 }
 

@@ -61,8 +61,17 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None, W_old=None):
     return out
 
 
+def default_vocab_chunk(V):
+    """The library's default vocabulary chunk without dW pairing: V split into
+    ceil(V / 32768) equal pieces rounded up to 256 columns (0 when that is one
+    piece, i.e. the whole vocabulary)."""
+    n = -(-V // 32768)
+    w = -(-(-(-V // n)) // 256) * 256
+    return 0 if w >= V else w
+
+
 def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_len=None,
-            keep_logits=False, pair_dw=False, W_old=None):
+            keep_logits=False, pair_dw=False, W_old=None, vocab_chunk=0):
     """Algorithm 1 inner loops through the C ABI; inputs already on `dev`.
 
     The old-policy pass is forward-only and keeps no logits; `keep_logits`
@@ -71,6 +80,7 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     `pair_dw` sets BGPO_FLAG_PAIR_DW for the inner loop in the same way.
     W_old (device bf16 [V, H]): the old-policy pass runs with this head and
     l_old is its output (no eps); otherwise l_old = l_self + eps.
+    vocab_chunk: bgpo_problem.vocab_chunk of the inner loop (0 = default).
 
     Returns dict of torch tensors: ell [B, n_t], ell_old, coef, g, t [n_t, B],
     masks [n_t, B, R], A, dX [B, R, H], dW [V, H], ws.
@@ -82,9 +92,10 @@ def gpu_run(wl, inp, dev="cuda", loss_scale=None, trace=None, b_offset=0, resp_l
     if resp_len is not None:
         lens = torch.as_tensor(np.asarray(resp_len), dtype=torch.int32, device=dev)
     prob = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                           resp_len=lens, keep_logits=keep_logits, pair_dw=pair_dw)
+                           resp_len=lens, keep_logits=keep_logits, pair_dw=pair_dw,
+                           vocab_chunk=vocab_chunk)
     prob_old = bg.problem_from(wl, trace=trace, loss_scale=loss_scale, b_offset=b_offset,
-                               resp_len=lens)
+                               resp_len=lens, vocab_chunk=vocab_chunk)
     ws = bg.alloc_workspace(prob, dev)
     bg.clear_device_error(ws)
     B, n_t = wl.B, wl.n_t

@@ -45,7 +45,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_names(L, bg):
-    assert L.bgpo_abi_version() == 2
+    assert L.bgpo_abi_version() == 3
     assert L.bgpo_status_string(0) == b"BGPO_OK"
     assert L.bgpo_status_string(8) == b"BGPO_ERR_TIMEOUT"
     assert L.bgpo_status_string(9) == b"BGPO_ERR_BOUNDS"
@@ -59,7 +59,7 @@ def test_problem_struct_layout(bg):
     assert bg.BgpoProblem.trace.offset == 48
     assert bg.BgpoProblem.resp_len.offset == 56
     assert bg.BgpoProblem.flags.offset == 64
-    assert bg.BgpoProblem.reserved.offset == 68
+    assert bg.BgpoProblem.vocab_chunk.offset == 68
 
 
 def _prob(bg, **kw):
@@ -99,8 +99,12 @@ def test_validation_of_flags(L, bg):
     assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
     p.flags = 0
-    p.reserved = 7
-    assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    for bad in (7, -256, 100, 255):        # vocab_chunk: a non-negative multiple of 256
+        p.vocab_chunk = bad
+        assert L.bgpo_validate_problem(ctypes.byref(p)) == 1
+    for good in (0, 256, 512, 1 << 24):
+        p.vocab_chunk = good
+        assert L.bgpo_validate_problem(ctypes.byref(p)) == 0
 
 
 def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
@@ -114,18 +118,44 @@ def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
         assert keep - lean == -(-4 * m_pad * v_pad // 1024) * 1024
 
 
-def test_pairing_doubles_only_dz_and_xm_transpose(L, bg):
-    # BGPO_FLAG_PAIR_DW gives dZ [rows, roundup(V, 64)] and Xm^T [H, rows] twice
-    # the rows: 2 * roundup(B R, 256) * (roundup(V, 64) + H) more bytes, with or
-    # without the logit region
-    for (B, R, V, H) in ((2, 32, 512, 64), (3, 301, 1000, 192), (16, 512, 126464, 4096)):
+def _default_chunk(V):
+    # default vocabulary chunk: V split into ceil(V / 32768) equal pieces rounded
+    # up to 256 columns; one piece is the whole vocabulary (roundup(V, 64))
+    n = -(-V // 32768)
+    w = -(-(-(-V // n)) // 256) * 256
+    return -(-V // 64) * 64 if w >= V else w
+
+
+def test_pairing_doubles_xm_transpose_and_keeps_dz_for_the_whole_vocabulary(L, bg):
+    # BGPO_FLAG_PAIR_DW gives Xm^T [H, rows] twice the rows and dZ twice the rows
+    # over the whole vocabulary (roundup(V, 64) columns) instead of one chunk:
+    # 2 m_pad H + 2 (2 m_pad v_pad - m_pad chunk) more bytes, with or without the
+    # logit region
+    for (B, R, V, H) in ((2, 32, 512, 64), (3, 301, 1000, 192), (16, 512, 126464, 4096),
+                         (32, 1024, 152064, 3584)):
         m_pad = -(-B * R // 256) * 256
         v_pad = -(-V // 64) * 64
         for keep in (False, True):
             lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep)))
             pair = L.bgpo_workspace_bytes(ctypes.byref(
                 _prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep, pair_dw=True)))
-            assert pair - lean == 2 * m_pad * (v_pad + H)
+            assert pair - lean == 2 * m_pad * H + 2 * (2 * m_pad * v_pad - m_pad * _default_chunk(V))
+
+
+def test_vocabulary_chunk_sets_the_dz_buffer(L, bg):
+    # dZ holds roundup(B R, 256) x chunk bf16 values: the default chunk, an
+    # explicit one, and the whole vocabulary (a chunk of V or more)
+    B, R, V, H = 16, 512, 126464, 4096
+    m_pad = B * R
+    assert _default_chunk(V) == 31744
+    size = lambda **kw: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, H=H, **kw)))
+    whole = size(vocab_chunk=1 << 17)
+    assert whole - size() == 2 * m_pad * (V - 31744)
+    assert whole - size(vocab_chunk=8192) == 2 * m_pad * (V - 8192)
+    assert size(vocab_chunk=V // 256 * 256 + 256) == whole
+    # with pairing the default keeps the whole vocabulary; an explicit chunk
+    # only sets how the backward walks it, not the buffer
+    assert size(pair_dw=True) == size(pair_dw=True, vocab_chunk=8192)
 
 
 def test_workspace_independent_of_n_t(L, bg):
@@ -144,13 +174,13 @@ def test_workspace_grows_with_rows_and_vocab(L, bg):
 def test_workspace_of_paper_shapes_fits_hbm(L, bg):
     # LLaDA-8B head, 16 x 512 responses; Dream-7B head, 32 x 1024 (bytes, not n_t-dependent)
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3)
-    assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 3e9
+    assert 0.5e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 1.5e9
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, keep_logits=True)
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 8e9
     p = bg.problem(16, 256, 512, 4096, 126464, 16, 8, 1, 3, pair_dw=True)
     assert 1e9 < L.bgpo_workspace_bytes(ctypes.byref(p)) < 5e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5)
-    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 16e9
+    assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 5e9
     p = bg.problem(32, 512, 1024, 3584, 152064, 16, 8, 0, 5, keep_logits=True)
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) < 40e9
 
@@ -251,5 +281,5 @@ def test_checked_build_exports_the_same_abi():
     for name, (res, args) in _lib.SIGNATURES.items():
         f = getattr(h, name)
         f.restype, f.argtypes = res, args
-    assert h.bgpo_abi_version() == 2
+    assert h.bgpo_abi_version() == 3
     assert h.bgpo_status_string(9) == b"BGPO_ERR_BOUNDS"

@@ -1,9 +1,11 @@
 """GPU parity at the size limits the C ABI accepts, one dimension at a time.
 
   * V = 2^24 - 1000 (just under the largest vocabulary, ragged against every
-    tile width): 65,532 vocabulary tiles in the forward and dW GEMMs, a 2^24-long
-    K loop in the dX GEMM, 64-bit offsets into dZ and the kept logits, and into
-    the paired dZ rows with BGPO_FLAG_PAIR_DW;
+    tile width): 65,532 vocabulary tiles in the forward GEMM, 512 vocabulary
+    chunks of 32,768 columns in the backward by default, and with
+    BGPO_FLAG_PAIR_DW one whole-vocabulary chunk (a 2^24-long K loop in the dX
+    GEMM, 65,532 vocabulary tiles in the dW GEMM); 64-bit offsets into dZ and
+    the kept logits, and into the paired dZ rows;
   * B * R = 2^22 (the most response positions): the single-CTA mask compaction
     walks 2^20 Philox blocks, about 2^21 masked rows per sample;
   * H = 16384 (the largest hidden size): 64 hidden-size tiles, 256 K blocks per
@@ -17,7 +19,8 @@ import pytest
 
 from oracle import bgpo_oracle as O
 from synth import CONFIGS, make_inputs
-from tests.harness import ensure_built, gpu_run, normwise, oracle_run, rel_ell_err, to64
+from tests.harness import (default_vocab_chunk, ensure_built, gpu_run, normwise, oracle_run,
+                           rel_ell_err, to64)
 
 pytestmark = pytest.mark.gpu
 
@@ -59,15 +62,26 @@ def test_largest_vocabulary(bg):
     assert torch.equal(k["dW"], g["dW"])
     del k
     # dW pairing puts sample 1's dZ rows after sample 0's (64-bit row offsets
-    # into a 2 * 256 x 2^24 bf16 region): same l and dX bits, dW up to order
-    q = gpu_run(wl, inp, pair_dw=True)
+    # into a 2 * 256 x 2^24 bf16 region); walking the vocabulary in the same
+    # 512 chunks as the unpaired backward: same l and dX bits, dW up to order
+    q = gpu_run(wl, inp, pair_dw=True, vocab_chunk=default_vocab_chunk(wl.V))
     assert bg.get_device_error(q["ws"]) == (0, 0)
     assert torch.equal(q["ell"], g["ell"]) and torch.equal(q["dX"], g["dX"])
     assert normwise(to64(q["dW"]), to64(g["dW"])) <= 1e-5
+    del q
+    # the pairing's default: the whole vocabulary in one chunk, i.e. one dX
+    # GEMM whose fp32 accumulator runs over K = 2^24 - 1000 vocabulary entries
+    # (the chunked one sums 512 chunk results): both against the oracle
+    q = gpu_run(wl, inp, pair_dw=True)
+    assert bg.get_device_error(q["ws"]) == (0, 0)
+    assert torch.equal(q["ell"], g["ell"])
+    q = {key: q[key].cpu() for key in ("masks", "t", "ell", "dX", "dW")}
     g = {key: g[key].cpu() for key in ("masks", "t", "ell", "dX", "dW")}
-    del q, inp
+    del inp
     torch.cuda.empty_cache()
-    _check(wl, g, oracle_run(wl, inp_cpu))
+    o = oracle_run(wl, inp_cpu)
+    _check(wl, g, o)
+    _check(wl, q, o)
 
 
 def test_most_response_positions(bg):

@@ -20,6 +20,9 @@ ELL_TOL = 1e-3
 GRAD_TOL = 2e-2
 # paired and unpaired dW differ only in the order of fp32 additions
 ORDER_TOL = 1e-5
+# dX summed over the whole LLaDA-8B vocabulary at once or in 4 chunks: fp32
+# order over a 126,464-long K whose terms mostly cancel (measured 2.0e-5)
+VOCAB_ORDER_TOL = 1e-4
 
 KID_MASK_COMPACT, KID_DW_GEMM = 0, 9
 
@@ -61,8 +64,12 @@ def test_paired_dw_matches_oracle_and_unpaired(bg, name, n_t, keep):
 
 def test_paired_dw_at_the_full_head(bg):
     """Full LLaDA-8B head (494 vocabulary tiles, K = 4096), 4 samples with few
-    masked rows each: the whole dW and dX against the oracle and the unpaired path."""
+    masked rows each: the whole dW and dX against the oracle and the unpaired
+    path. The unpaired backward walks the vocabulary in 4 chunks by default,
+    the paired one in 1 (its dZ holds the whole vocabulary): the same dX up to
+    fp32 order; walked in the same chunks, the same dX bits."""
     import torch
+    from tests.harness import default_vocab_chunk
     wl = CONFIGS["llada8b_r256"].with_(B=2, P=8, R=24, n_t=4, G=2)
     inp_cpu = make_inputs(wl)
     inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
@@ -71,9 +78,14 @@ def test_paired_dw_at_the_full_head(bg):
     res = {k: p[k].cpu() for k in ("masks", "ell", "dX", "dW")}
     del p
     a = gpu_run(wl, inp)
-    assert torch.equal(res["ell"], a["ell"].cpu()) and torch.equal(res["dX"], a["dX"].cpu())
+    assert torch.equal(res["ell"], a["ell"].cpu())
+    assert normwise(to64(res["dX"]), to64(a["dX"])) <= VOCAB_ORDER_TOL
     assert normwise(to64(res["dW"]), to64(a["dW"])) <= ORDER_TOL
-    del a
+    c = gpu_run(wl, inp, pair_dw=True, vocab_chunk=default_vocab_chunk(wl.V))
+    assert bg.get_device_error(c["ws"]) == (0, 0)
+    assert torch.equal(c["ell"], a["ell"]) and torch.equal(c["dX"], a["dX"])
+    assert normwise(to64(c["dW"]), to64(a["dW"])) <= ORDER_TOL
+    del a, c
     torch.cuda.empty_cache()
     o = oracle_run(wl, inp_cpu)
     assert np.array_equal(res["masks"].numpy(), o["masks"])

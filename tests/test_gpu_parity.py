@@ -273,8 +273,20 @@ def test_trace_records_every_kernel(bg):
     bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
     names = [n for n, ms in tr.records()]
     assert names == ["mask_compact", "gather_rows", "lmhead_fwd_lse", "lse_combine", "seq_reduce",
-                     "bound_coeffs", "lmhead_dz", "dx_gemm", "dx_reduce", "xm_transpose", "dw_gemm"]
+                     "bound_coeffs", "xm_transpose", "lmhead_dz", "dx_gemm", "dx_reduce", "dw_gemm"]
     assert all(ms >= 0 for _, ms in tr.records())
+    tr.close()
+    # the backward over two vocabulary chunks of 256 columns: each chunk's dZ,
+    # dX and dW GEMMs, then one split reduction of dX
+    tr = bg.Trace(64)
+    p = bg.problem_from(wl, trace=tr, vocab_chunk=256)
+    ws = bg.alloc_workspace(p)
+    bg.sample_mask(p, 0, ws)
+    bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
+    bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
+    assert [n for n, ms in tr.records()][5:] == ["xm_transpose"] + 2 * ["lmhead_dz", "dx_gemm",
+                                                                        "dw_gemm"] + ["dx_reduce"]
+    assert bg.get_device_error(ws) == (0, 0)
     tr.close()
     # with BGPO_FLAG_KEEP_LOGITS the backward reads the logits the forward kept
     tr = bg.Trace(64)
@@ -283,8 +295,8 @@ def test_trace_records_every_kernel(bg):
     bg.sample_mask(p, 0, ws)
     bg.elbo_fwd(p, 0, inp["X"], inp["W"], inp["Y"], ws, ell)
     bg.elbo_bwd_accumulate(p, 0, inp["X"], inp["W"], inp["Y"], coef, ws, dX, dW)
-    assert [n for n, ms in tr.records()][-5:] == ["dz_from_logits", "dx_gemm", "dx_reduce",
-                                                  "xm_transpose", "dw_gemm"]
+    assert [n for n, ms in tr.records()][-5:] == ["xm_transpose", "dz_from_logits", "dx_gemm",
+                                                  "dx_reduce", "dw_gemm"]
     assert bg.get_device_error(ws) == (0, 0)
     tr.close()
 

@@ -26,17 +26,20 @@ static void layout(int64_t B, int64_t R, int64_t H, int64_t V) {
   const Geometry g = make_geometry(B, 1, R, H, V);
   for (int keep = 0; keep < 2; ++keep)
     for (int pair = 0; pair < 2; ++pair) {
-      const WsLayout L = make_ws_layout(g, keep, pair);
+      const Geometry gp = make_geometry(B, 1, R, H, V, 0, pair);
+      const WsLayout L = make_ws_layout(gp, keep, pair);
       printf("{\"kind\": \"layout\", \"B\": %lld, \"R\": %lld, \"H\": %lld, \"V\": %lld, "
              "\"keep\": %d, \"pair\": %d, \"off\": [%zu, %zu, %zu, %zu, %zu, %zu, %zu, %zu, %zu, "
              "%zu, %zu, %zu, %zu, %zu, %zu], \"dz_rows\": %zu, \"dxp_elems\": %zu, "
              "\"zc_bytes\": %zu, \"total\": %zu, \"cap\": %lld, \"fwd\": %zu, \"m_pad\": %lld, "
-             "\"n_vt\": %lld}\n",
+             "\"n_vt\": %lld, \"dz_cols\": %zu, \"local\": %d, \"vc\": %lld, \"n_vc\": %lld, "
+             "\"kb_vc_min\": %lld}\n",
              (long long)B, (long long)R, (long long)H, (long long)V, keep, pair, L.err, L.t,
              L.tnum, L.seg_off, L.rows, L.tgt, L.tgt_logit, L.lse, L.logp, L.part, L.xm, L.xmT,
              L.dz, L.dxp, L.zc, L.dz_rows, L.dxp_elems, L.zc_bytes, L.total,
-             (long long)dxp_row_block_cap(g), L.fwd_bytes, (long long)g.m_pad,
-             (long long)g.n_vt);
+             (long long)dxp_row_block_cap(gp), L.fwd_bytes, (long long)gp.m_pad,
+             (long long)gp.n_vt, L.dz_cols, (int)L.dz_chunk_local, (long long)gp.vc,
+             (long long)gp.n_vc, (long long)gp.kb_vc_min);
     }
   const int64_t cap = dxp_row_block_cap(g);
   for (int64_t mb = 1; mb <= g.m_pad / kPairM; ++mb)
@@ -102,7 +105,7 @@ def test_workspace_regions_fit_in_order(plan):
         need = {"err": 64, "t": 4 * B, "tnum": 8 * B, "seg_off": 4 * (B + 1), "rows": 4 * m_cap,
                 "tgt": 4 * m_pad, "tgt_logit": 4 * m_pad, "lse": 4 * m_pad, "logp": 4 * m_pad,
                 "part": 8 * m_pad * n_vt, "xm": 2 * m_pad * H, "xmT": 2 * H * dz_rows,
-                "dz": 2 * dz_rows * v_pad, "dxp": 4 * L["dxp_elems"],
+                "dz": 2 * dz_rows * L["dz_cols"], "dxp": 4 * L["dxp_elems"],
                 "zc": 4 * m_pad * v_pad if L["keep"] else 0}
         # the split buffer holds cap row blocks of 256 rows x H
         assert L["dxp_elems"] == L["cap"] * 256 * H
@@ -175,3 +178,22 @@ def test_forward_regions_fit_the_documented_bound(plan):
         assert L["off"][10] < L["fwd"] <= bound           # xm starts below the end
         assert L["fwd"] == L["off"][11]                    # Xm^T starts where it ends
         assert L["fwd"] % 1024 == 0
+
+
+def test_vocabulary_chunks(plan):
+    # default chunks: V split evenly into ceil(V / 32768) pieces rounded up to
+    # 256 columns (one piece: the whole vocabulary, roundup(V, 64)); with dW
+    # pairing one chunk; dZ holds one chunk unless it must hold them all
+    for L in plan["layout"]:
+        V = L["V"]
+        v_pad = _ceil(V, 64) * 64
+        n = _ceil(V, 32768)
+        w = _ceil(_ceil(V, n), 256) * 256
+        vc = v_pad if (L["pair"] or w >= V) else w
+        assert L["vc"] == vc and L["n_vc"] == _ceil(V, vc)
+        assert (L["n_vc"] - 1) * vc < V <= L["n_vc"] * vc
+        last = V - (L["n_vc"] - 1) * vc
+        assert L["kb_vc_min"] == _ceil(min(last, vc), 64)
+        assert L["local"] == int(L["n_vc"] > 1 and not L["pair"])
+        assert L["dz_cols"] == (vc if L["local"] else v_pad)
+        assert vc % 256 == 0 or vc == v_pad

@@ -4,8 +4,9 @@ Every (sequence, MC sample) unit is independent once A and l_old are given
 (Linearity, Sec. 3), so the path shards by sequences with no collective in the
 data path; the dW sum over ranks belongs to the optimiser step. Two gloo ranks
 each run the fp64 oracle on their half of a batch (b_offset = first global
-sequence index), all-reduce dW and gather dX and l; rank 0 compares with the
-single-process run of the whole batch. The bench's rank aggregation (slowest
+sequence index), sum dW with the bench's data-parallel exchange
+(paper_2510_11683_gb300.dp.allreduce_dw) and gather dX and l; rank 0 compares
+with the single-process run of the whole batch. The bench's rank aggregation (slowest
 rank's time, tokens of all ranks) is checked on the same ranks.
 """
 import os
@@ -18,6 +19,7 @@ import torch.distributed as dist
 import torch.multiprocessing as mp
 
 from oracle import bgpo_oracle as O
+from paper_2510_11683_gb300.dp import allreduce_dw
 from synth import CONFIGS, make_inputs
 from tests.harness import oracle_advantages, to64
 
@@ -51,7 +53,7 @@ def _rank_main(rank, port, out_dir):
         ell_old = O.elbo_all(X, W, Y, wl.P, ts, masks) + eps
         out = O.bgpo_step(X, W, Y, wl.P, A, ell_old, ts, masks, 1.0 / wl.G)
         dW = torch.from_numpy(out["dW"])
-        dist.all_reduce(dW)                        # the optimiser step's gradient sum
+        allreduce_dw(dW)                           # the optimiser step's gradient sum
         dX = [torch.zeros_like(torch.from_numpy(out["dX"])) for _ in range(WORLD)]
         dist.all_gather(dX, torch.from_numpy(out["dX"]))
         ell = [torch.zeros_like(torch.from_numpy(out["ell"])) for _ in range(WORLD)]
@@ -117,7 +119,7 @@ def _lost_rank_main(rank, port, out_dir):
         return                                     # leaves without joining the sum
     dW = torch.from_numpy(out["dW"])
     try:
-        dist.all_reduce(dW)
+        allreduce_dw(dW)
         result = "completed"
     except Exception as e:                         # noqa: BLE001 - any collective failure
         result = "detected: " + type(e).__name__
@@ -133,3 +135,10 @@ def test_lost_rank_is_detected_by_the_survivor(tmp_path):
         result = f.read()
     assert result.startswith("detected"), result
     assert time.time() - t0 < 120
+
+
+def test_single_process_exchange_is_the_identity():
+    # without an initialised process group there is nothing to sum over
+    dW = torch.arange(12, dtype=torch.float32).reshape(3, 4)
+    ref = dW.clone()
+    assert allreduce_dw(dW) is dW and torch.equal(dW, ref)
