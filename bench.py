@@ -46,15 +46,17 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind, mean
-# over one step of the bench workload with dW paired, from one single-pass ncu
-# capture of that step. Valid only for that workload and mode, and while the
-# GEMM sources hash to `sha` (otherwise the line reports traffic as null).
+# dram__bytes_read.sum + dram__bytes_write.sum of the forward and dZ GEMMs per
+# 256 x 256 pair tile, from ncu captures of single launches on the small case
+# llada8b_r512_b8 (MC samples 12 and 13, 13 and 14 row blocks x 494 vocabulary
+# tiles, dW paired as in the bench step); a launch's traffic is scaled by its
+# pair tiles. Valid while the GEMM sources hash to `sha` (otherwise the line
+# reports traffic as null); the dX and dW GEMMs' traffic is not proportional to
+# their tiles and is not estimated.
 TRAFFIC = {
-    "workload": "llada8b_r512_onpolicy",
-    "sha": "10549a8464f33f9257c851e45de86d1a6ef464b6a5eb06635362b13a27d7693e",
-    "bytes_per_launch": {"lmhead_fwd_lse": 2.0363e+09, "lmhead_dz": 3.9066e+09,
-                          "dx_gemm": 7.5147e+09, "dw_gemm": 1.5873e+10},
+    "sha": "f6588a6ec6612107068d29bdc644ed9d2fdede82593cf02d4c8a8cc593940d71",
+    "bytes_per_tile": {"lmhead_fwd_lse": 1.65e5, "lmhead_dz": 3.16e5},
+    "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by pair tiles",
 }
 
 
@@ -76,6 +78,14 @@ def parse():
                     help="skip the unpaired leg with the whole vocabulary as one chunk")
     ap.add_argument("--grad-variance", action="store_true",
                     help="run the Sec. 4.3 gradient std / bias vs n_t study instead")
+    ap.add_argument("--profile-sample", type=int, default=None, metavar="J",
+                    help="run MC sample J's path once (mask, forward, coefficients, backward; "
+                         "with dW paired and J odd, sample J - 1 first) and exit: a short "
+                         "process whose kernels ncu can capture after few launches")
+    ap.add_argument("--vocab-chunk", type=int, default=0,
+                    help="bgpo_problem.vocab_chunk for --profile-sample (0 = default)")
+    ap.add_argument("--keep", action="store_true",
+                    help="BGPO_FLAG_KEEP_LOGITS for --profile-sample")
     return ap.parse_args()
 
 
@@ -273,6 +283,9 @@ def main():
     if args.grad_variance:
         run_grad_variance(args, CONFIGS["llada8b_sweep"] if args.workload == WORKLOAD else wl)
         return
+    if args.profile_sample is not None:
+        run_profile_sample(args, wl)
+        return
 
     import torch
     rank, world, local = dist_env()
@@ -394,11 +407,14 @@ def main():
         dom_avg_s = dom_ms / dom_launches / 1e3
         achieved = dom_flops_per_launch / dom_avg_s / 1e12
         traffic = None
-        if (headline_mode and wl.name == TRAFFIC["workload"] and TRAFFIC["sha"] == kernel_sha()
-                and world == 1):
-            traffic = TRAFFIC["bytes_per_launch"].get(dom)
+        per_tile = TRAFFIC["bytes_per_tile"].get(dom)
+        if headline_mode and per_tile and TRAFFIC["sha"] == kernel_sha():
+            # pair tiles per launch: row blocks of each sample x vocabulary tiles
+            tiles = sum(-(-m // 256) for m in rows_per_sample) * (-(-V // 256)) / n_t
+            traffic = per_tile * tiles
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
+                "traffic_source": TRAFFIC["source"] if traffic is not None else None,
                 "kernel": dom, "peak_kind": f"bf16 sustained ({peaks['source']})",
                 "flops_per_launch": dom_flops_per_launch, "avg_launch_ms": dom_avg_s * 1e3}
         # dL/dz from kept logits: reads 4 V and writes 2 V bytes per masked row
@@ -597,6 +613,45 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     return {"value": masked_per_step / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps,
             "pipelining": "inputs of step k+1 copied on a second stream during step k"}
+
+
+def run_profile_sample(args, wl):
+    """One MC sample's path through the C ABI with as few launches as possible
+    before it: inputs, advantages, then mask, forward, coefficients (on-policy,
+    d = 0) and backward of sample J (of J - 1 and J when dW is paired and J is
+    odd). Prints the masked rows and the device error word per sample."""
+    import torch
+    import paper_2510_11683_gb300 as bg
+    from paper_2510_11683_gb300 import build as B
+    from synth import make_inputs
+    if not os.path.exists(B.LIB_PATH):
+        B.build()
+    pair = not args.no_pair_dw
+    inp = make_inputs(wl, device="cuda")
+    X, W, Y = inp["X"], inp["W"], inp["Y"]
+    p = bg.problem_from(wl, pair_dw=pair, keep_logits=args.keep, vocab_chunk=args.vocab_chunk)
+    ws = bg.alloc_workspace(p)
+    A = torch.empty(wl.B, dtype=torch.float32, device="cuda")
+    if inp["A"] is not None:
+        A.copy_(inp["A"])
+    else:
+        bg.group_advantage(p, inp["rewards"], A)
+    ell = torch.empty(wl.B, dtype=torch.float32, device="cuda")
+    coef = torch.empty_like(ell)
+    dX = torch.zeros((wl.B, wl.R, wl.H), dtype=torch.float32, device="cuda")
+    dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device="cuda")
+    m = torch.empty((wl.B, wl.R), dtype=torch.uint8, device="cuda")
+    j = args.profile_sample
+    for jj in ([j - 1, j] if pair and j % 2 == 1 else [j]):
+        bg.sample_mask(p, jj, ws, None, m)
+        bg.elbo_fwd(p, jj, X, W, Y, ws, ell)
+        bg.bound_coeffs(p, jj, ell, ell, A, coef, None, ws)
+        bg.elbo_bwd_accumulate(p, jj, X, W, Y, coef, ws, dX, dW)
+        torch.cuda.synchronize()
+        print(json.dumps({"sample": jj, "masked_rows": int(m.sum()),
+                          "device_error": list(bg.get_device_error(ws))}), flush=True)
+    print(json.dumps({"workspace_bytes": ws.numel(),
+                      "peak_mem_bytes": torch.cuda.max_memory_allocated()}), flush=True)
 
 
 def grad_seed(wl, n_t, rep):

@@ -31,7 +31,7 @@
  *  - Layouts are dense row-major: X [B, P+R, H], W [V, H], Y [B, R],
  *    dX [B, R, H] (response rows only), dW [V, H], per-sequence vectors [B].
  *  - Alignment: X, W, dX, dW and the workspace must be 16-byte aligned
- *    (workspace: 256-byte). H must be a multiple of 64.
+ *    (workspace: 256-byte). H must be a multiple of 8 (16-byte rows of X and W).
  *  - The workspace carries sample j's draws (t, mask), its compacted masked
  *    rows, forward statistics and (with BGPO_FLAG_KEEP_LOGITS) the masked
  *    rows' logits from one call to the next, so the calls for
@@ -132,7 +132,8 @@ typedef struct bgpo_trace bgpo_trace;
  *   B      responses in the batch (>= 1)
  *   P      prompt length: X rows [b, 0, P) are the prompt, never masked (Sec. 2.1)
  *   R      response length (>= 1); response position i is X row [b, P + i]
- *   H      hidden size, multiple of 64, 64 <= H <= 16384
+ *   H      hidden size, multiple of 8, 64 <= H <= 16384 (a last K block or hidden-size
+ *          tile that H does not fill is read as zeros and written only up to H)
  *   V      vocabulary size, 1 <= V <= 2^24
  *   n_t    MC samples per response, 1 <= n_t < 65536 (Eq. 5)
  *   G      group size used by bgpo_group_advantage (Eq. 18), >= 1

@@ -68,7 +68,7 @@ bgpo_status check_problem(const bgpo_problem* p) {
   if ((p->flags & ~(BGPO_FLAG_KEEP_LOGITS | BGPO_FLAG_PAIR_DW)) != 0u) return BGPO_ERR_INVALID_ARG;
   if (p->vocab_chunk < 0 || p->vocab_chunk % kBN != 0) return BGPO_ERR_INVALID_ARG;
   if (p->B < 1 || p->P < 0 || p->R < 1 || p->V < 1 || p->n_t < 1 || p->G < 1) return BGPO_ERR_SHAPE;
-  if (p->H < 64 || p->H % 64 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
+  if (p->H < 64 || p->H % 8 != 0 || p->H > kMaxH) return BGPO_ERR_SHAPE;
   if (p->V > kMaxV || p->n_t >= 65536) return BGPO_ERR_SHAPE;
   if ((int64_t)p->B * p->R > kMaxRows) return BGPO_ERR_SHAPE;
   if ((int64_t)p->b_offset + p->B > (int64_t(1) << 31)) return BGPO_ERR_SHAPE;

@@ -88,7 +88,8 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
     w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = KIND == GEMM_FWD ? p.g.n_vt : ceil_div(p.v_end - p.v_begin, kBN);
-    w.kb_total = p.g.H / kBK;
+    // a last K block past H reads the tensor maps' zero fill
+    w.kb_total = ceil_div(p.g.H, kBK);
     w.units = w.tiles_m * w.tiles_n;
   } else if (KIND == GEMM_DX) {
     w.tiles_m = ceil_div(M, kPairM);
@@ -405,6 +406,7 @@ __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* m
   const int32_t prow0 = (int32_t)(t.split * wk.tiles_m * kPairM + row0);
   const int64_t r = row0 + lane;
   float4* drow = nullptr;
+  const int32_t H = (int32_t)p.g.H;
   if (wk.splits == 1 && r < M &&
       BGPO_IN_BOUNDS(p.w.err, p.w.rows[r] >= 0 && p.w.rows[r] < p.g.m_cap, KID_DX_GEMM * 16 + 10))
     drow = reinterpret_cast<float4*>(p.dX + (int64_t)p.w.rows[r] * p.g.H + h0);
@@ -416,8 +418,11 @@ __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* m
     tmem_ld_wait();
     if (wk.splits == 1) {  // launch-uniform
       if (drow) {
+        // 16-byte pieces of this sub-tile inside the row (H is a multiple of 8)
+        const int nq = min(8, (H - (h0 + c * 32)) / 4);
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
+          if (q >= nq) break;
           float4 o = drow[c * 8 + q];
           o.x += bits_f(raw[4 * q]);
           o.y += bits_f(raw[4 * q + 1]);

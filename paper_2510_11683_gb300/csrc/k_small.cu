@@ -472,7 +472,10 @@ __global__ void __launch_bounds__(kTrThreads) k_xm_transpose(Geometry g, int32_t
 #pragma unroll
   for (int i = 0; i < kTrChunks; ++i) {   // chunk c: row c / 8, columns (c % 8) * 8 ..
     const int c = threadIdx.x + i * kTrThreads;
-    v[i] = *reinterpret_cast<const uint4*>(xm + (r0 + c / 8) * g.H + h0 + (c % 8) * 8);
+    // H is a multiple of 8: a chunk lies wholly inside or wholly past the row
+    v[i] = h0 + (c % 8) * 8 < g.H
+               ? *reinterpret_cast<const uint4*>(xm + (r0 + c / 8) * g.H + h0 + (c % 8) * 8)
+               : make_uint4(0, 0, 0, 0);
   }
 #pragma unroll
   for (int i = 0; i < kTrChunks; ++i) {
@@ -488,6 +491,7 @@ __global__ void __launch_bounds__(kTrThreads) k_xm_transpose(Geometry g, int32_t
     const int c = threadIdx.x + i * kTrThreads;
     const int hh = (c / 8) % kTrCols;
     const int rr = (c / (8 * kTrCols)) * 64 + (c % 8) * 8;
+    if (h0 + hh >= g.H) continue;     // Xm^T has H rows
     uint32_t word[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
@@ -624,7 +628,7 @@ cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, floa
 
 cudaError_t launch_xm_transpose(const Geometry& g, int32_t j, bool defer, const WsPtrs& w,
                                 cudaStream_t s) {
-  const dim3 grid((unsigned)(g.m_pad / kTrRows), (unsigned)(g.H / kTrCols));
+  const dim3 grid((unsigned)(g.m_pad / kTrRows), (unsigned)ceil_div(g.H, kTrCols));
   k_xm_transpose<<<grid, kTrThreads, 0, s>>>(g, j, defer, w);
   return cudaGetLastError();
 }

@@ -69,7 +69,8 @@ def _prob(bg, **kw):
 
 
 @pytest.mark.parametrize("kw,status", [
-    (dict(B=0), 2), (dict(R=0), 2), (dict(P=-1), 2), (dict(H=96), 2), (dict(H=0), 2),
+    (dict(B=0), 2), (dict(R=0), 2), (dict(P=-1), 2), (dict(H=100), 2), (dict(H=0), 2),
+    (dict(H=56), 2), (dict(H=16392), 2),
     (dict(V=0), 2), (dict(n_t=0), 2), (dict(n_t=65536), 2), (dict(G=0), 2),
     (dict(t_mode=2), 1), (dict(B=1 << 12, R=1 << 11), 2), (dict(V=(1 << 24) + 1), 2),
 ])
@@ -77,6 +78,12 @@ def test_validation_rejects_bad_problems(L, bg, kw, status):
     p = _prob(bg, **kw)
     assert L.bgpo_validate_problem(ctypes.byref(p)) == status
     assert L.bgpo_workspace_bytes(ctypes.byref(p)) == 0
+
+
+def test_hidden_sizes_in_16_byte_rows_are_accepted(L, bg):
+    # H needs 16-byte rows of bf16 (a multiple of 8) and at least one 64-wide K block
+    for H in (64, 72, 96, 200, 3584, 4104, 16384):
+        assert L.bgpo_validate_problem(ctypes.byref(_prob(bg, H=H))) == 0, H
 
 
 def test_validation_rejects_bad_offset_and_nonfinite_scale(L, bg):

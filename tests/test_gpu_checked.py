@@ -3,9 +3,12 @@
 The library ships a build whose kernels test every index they read from device
 memory (masked-row lists, segment offsets, row counts) and every target token
 before use, recording BGPO_ERR_BOUNDS instead of touching memory out of bounds:
-a memory checker built into the library, usable where no external one runs. Here the parity workloads run through that build, in a child process
-that loads it (BGPO_LIBRARY=checked): the error word must stay clear and the
-results must match the oracle as the normal build's do, in both logit modes.
+a memory checker built into the library, usable where no external one runs.
+Here the parity workloads run through that build, in a child process that
+loads it (BGPO_LIBRARY=checked): the error word must stay clear and the
+results must match the oracle as the normal build's do, in both logit modes
+and with the backward walking vocabulary chunks of 256 columns (with and
+without dW pairing).
 A target token outside the vocabulary, which the normal build cannot see (it
 only ever compares targets, never indexes with them), must be reported.
 """
@@ -42,9 +45,14 @@ def _child():
         inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
         g = gpu_run(wl, inp)
         k = gpu_run(wl, inp, keep_logits=True)
+        # the backward over vocabulary chunks of 256 columns, unpaired and paired
+        c = gpu_run(wl, inp, vocab_chunk=256)
+        q = gpu_run(wl, inp, pair_dw=True, vocab_chunk=256)
         o = oracle_run(wl, inp_cpu)
         out["parity"][name] = {
-            "errors": [bg.get_device_error(g["ws"]), bg.get_device_error(k["ws"])],
+            "errors": [bg.get_device_error(r["ws"]) for r in (g, k, c, q)],
+            "chunked": [max(normwise(to64(r["dX"]), o["dX"]), normwise(to64(r["dW"]), o["dW"]))
+                        for r in (c, q)],
             "masks": bool(np.array_equal(g["masks"].cpu().numpy(), o["masks"])),
             "ell": float(rel_ell_err(to64(g["ell"]), o["ell"]).max()),
             "dX": normwise(to64(g["dX"]), o["dX"]), "dW": normwise(to64(g["dW"]), o["dW"]),
@@ -71,7 +79,8 @@ def test_checked_build_runs_clean_and_reports_a_bad_target():
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
     res = json.loads(r.stdout.strip().splitlines()[-1])
     for name, p in res["parity"].items():
-        assert p["errors"] == [[0, 0], [0, 0]], (name, p)
+        assert p["errors"] == [[0, 0]] * 4, (name, p)
+        assert max(p["chunked"]) <= GRAD_TOL, (name, p)
         assert p["masks"], name
         assert p["ell"] <= ELL_TOL, (name, p)
         assert p["dX"] <= GRAD_TOL and p["dW"] <= GRAD_TOL, (name, p)

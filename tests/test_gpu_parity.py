@@ -414,14 +414,16 @@ def test_variable_length_responses(bg, keep, pair):
     assert float(g["dX"][2, 117:].abs().max()) == 0.0
 
 
-@pytest.mark.parametrize("keep,pair", [(False, False), (True, False), (False, True), (True, True)])
-def test_whole_step_replays_from_a_cuda_graph(bg, keep, pair):
+@pytest.mark.parametrize("keep,pair,chunk", [(False, False, 0), (True, False, 0), (False, True, 0),
+                                             (True, True, 0), (False, False, 256),
+                                             (True, True, 256)])
+def test_whole_step_replays_from_a_cuda_graph(bg, keep, pair, chunk):
     # the n_t loop allocates nothing, never synchronises and keeps M (and the
     # dW pairing state) on the device, so one step captures into a CUDA graph;
-    # a replay gives the bits of the eager step
+    # a replay gives the bits of the eager step (also over vocabulary chunks)
     import torch
     wl, inp = _inputs("ragged")
-    p = bg.problem_from(wl, keep_logits=keep, pair_dw=pair)
+    p = bg.problem_from(wl, keep_logits=keep, pair_dw=pair, vocab_chunk=chunk)
     X, W, Y = inp["X"], inp["W"], inp["Y"]
     ws = bg.alloc_workspace(p)
     A = inp["A"].contiguous()
@@ -503,3 +505,23 @@ def test_peak_device_memory_flat_in_n_t(bg, pair):
         del g, inp
     vectors = 16 * 4 * wl.B * 8          # [n_t, B] float vectors of the harness, generously
     assert peaks[16] - peaks[1] <= vectors + (1 << 20), peaks
+
+
+@pytest.mark.parametrize("H", [72, 200, 328])
+def test_hidden_sizes_not_a_multiple_of_64(bg, H):
+    """H a multiple of 8 only: the forward and dZ GEMMs end on a partial K
+    block (read as zeros), the dX and dW GEMMs on a partial hidden-size tile
+    and 32-column sub-tile (8 columns of H = 200, 72 and 328), the transpose
+    on a partial 64-column tile; with and without vocabulary chunks and dW
+    pairing."""
+    wl = CONFIGS["ragged"].with_(name="odd_hidden", H=H, seed=90 + H)
+    inp_cpu = make_inputs(wl)
+    inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
+    o = oracle_run(wl, inp_cpu)
+    for kw in (dict(), dict(vocab_chunk=256), dict(pair_dw=True), dict(keep_logits=True)):
+        g = gpu_run(wl, inp, **kw)
+        assert bg.get_device_error(g["ws"]) == (0, 0), kw
+        assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+        assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= ELL_TOL, kw
+        assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL, kw
+        assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL, kw
