@@ -55,7 +55,7 @@ UNIT = "tokens/s"
 # their tiles and is not estimated.
 TRAFFIC = {
     "sha": "f6588a6ec6612107068d29bdc644ed9d2fdede82593cf02d4c8a8cc593940d71",
-    "bytes_per_tile": {"lmhead_fwd_lse": 1.65e5, "lmhead_dz": 3.16e5},
+    "bytes_per_tile": {"lmhead_fwd_lse": 1.67e5, "lmhead_dz": 3.41e5},
     "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by pair tiles",
 }
 
