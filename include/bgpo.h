@@ -156,10 +156,12 @@ typedef struct bgpo_trace bgpo_trace;
  *          buffer in the workspace holds roundup(B R, 256) x vocab_chunk
  *          bf16 values instead of roundup(B R, 256) x V (Linearity, Sec. 3: the
  *          gradient is a sum over vocabulary entries as well as over samples).
- *          Default: chunks of at most 32768 columns (V split evenly, rounded
- *          up to 256); with BGPO_FLAG_PAIR_DW, whose even samples leave their
- *          dL/dz for the whole vocabulary pending, one chunk. A chunk of V or
- *          more columns is the whole vocabulary at once. l and dW are the same
+ *          Default: the whole vocabulary at once when its dL/dz takes at most
+ *          1 GiB (2 roundup(B R, 256) roundup(V, 64) bytes) or with
+ *          BGPO_FLAG_PAIR_DW (whose even samples leave their dL/dz for the
+ *          whole vocabulary pending); otherwise chunks of at most 32768
+ *          columns (V split evenly, rounded up to 256). A chunk of V or more
+ *          columns is the whole vocabulary at once. l and dW are the same
  *          bits for every chunk width; dX is the same sum up to fp32 order.
  * B * R must not exceed 2^22 and B * R * V must fit the workspace (see
  * bgpo_workspace_bytes).

@@ -29,6 +29,10 @@ constexpr int kMaxSplits = 16;   // split-K limit of the dX GEMM
 // the dX GEMM and the dW GEMM one chunk of at most this many columns at a
 // time, so its buffer holds M x V_c instead of M x V.
 constexpr int64_t kVChunkDefault = 32768;
+// By default the vocabulary is walked in one piece when dZ for the whole of it
+// takes at most this many bytes: chunks then save little memory and their
+// launch tails cost most (few masked rows per launch).
+constexpr int64_t kDzWholeMaxBytes = int64_t(1) << 30;
 
 constexpr uint32_t kTileABytes = kBM * kBK * 2;       // 16 KB per CTA
 constexpr uint32_t kTileBBytes = kBNHalf * kBK * 2;   // 16 KB per CTA
@@ -86,15 +90,16 @@ BGPO_HD int dx_splits(int64_t mb, int64_t tiles_n, int num_pairs, int64_t k_bloc
 }
 
 // Width of the backward's vocabulary chunks. `request` 0 asks for the
-// default: one chunk when dW pairing keeps the whole vocabulary's dZ anyway,
-// else the V columns split into ceil(V / kVChunkDefault) chunks of equal
-// width rounded up to a tile. A positive request is a multiple of kBN (the
-// host validates it). A width of V or more is a single chunk.
-BGPO_HD int64_t vocab_chunk_width(int64_t V, int64_t request, bool pair_dw) {
+// default: one chunk when dW pairing keeps the whole vocabulary's dZ anyway or
+// when that dZ (m_pad rows of roundup(V, 64) bf16 values) fits
+// kDzWholeMaxBytes, else the V columns split into ceil(V / kVChunkDefault)
+// chunks of equal width rounded up to a tile. A positive request is a multiple
+// of kBN (the host validates it). A width of V or more is a single chunk.
+BGPO_HD int64_t vocab_chunk_width(int64_t V, int64_t request, bool pair_dw, int64_t m_pad) {
   int64_t w;
   if (request > 0) {
     w = request;
-  } else if (pair_dw) {
+  } else if (pair_dw || 2 * m_pad * round_up(V, 64) <= kDzWholeMaxBytes) {
     w = V;
   } else {
     const int64_t n = ceil_div(V, kVChunkDefault);
@@ -127,7 +132,7 @@ BGPO_HD Geometry make_geometry(int64_t B, int64_t P, int64_t R, int64_t H, int64
   g.n_vt = ceil_div(V, kBN);
   g.tiles_h = ceil_div(H, kBN);
   g.kb_v = ceil_div(V, kBK);
-  g.vc = vocab_chunk_width(V, vchunk_request, pair_dw);
+  g.vc = vocab_chunk_width(V, vchunk_request, pair_dw, g.m_pad);
   g.n_vc = ceil_div(V, g.vc);
   const int64_t last = V - (g.n_vc - 1) * g.vc;
   g.kb_vc_min = ceil_div(last < g.vc ? last : g.vc, kBK);

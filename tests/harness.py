@@ -61,10 +61,14 @@ def oracle_run(wl, inp, loss_scale=None, b_offset=0, resp_len=None, W_old=None):
     return out
 
 
-def default_vocab_chunk(V):
-    """The library's default vocabulary chunk without dW pairing: V split into
-    ceil(V / 32768) equal pieces rounded up to 256 columns (0 when that is one
-    piece, i.e. the whole vocabulary)."""
+def default_vocab_chunk(V, rows=None):
+    """The library's chunk width without dW pairing for a vocabulary V split
+    into ceil(V / 32768) equal pieces rounded up to 256 columns (0 when that
+    is one piece). With `rows` = B R, the default proper: 0 (the whole
+    vocabulary) also when its dL/dz, roundup(rows, 256) x roundup(V, 64) bf16
+    values, takes at most 1 GiB."""
+    if rows is not None and 2 * (-(-rows // 256) * 256) * (-(-V // 64) * 64) <= 1 << 30:
+        return 0
     n = -(-V // 32768)
     w = -(-(-(-V // n)) // 256) * 256
     return 0 if w >= V else w

@@ -125,12 +125,16 @@ def test_logit_region_is_the_only_difference_of_the_flag(L, bg):
         assert keep - lean == -(-4 * m_pad * v_pad // 1024) * 1024
 
 
-def _default_chunk(V):
-    # default vocabulary chunk: V split into ceil(V / 32768) equal pieces rounded
-    # up to 256 columns; one piece is the whole vocabulary (roundup(V, 64))
+def _default_chunk(V, m_pad):
+    # default vocabulary chunk: the whole vocabulary (roundup(V, 64)) when its
+    # dZ, m_pad x roundup(V, 64) bf16, fits 1 GiB; else V split into
+    # ceil(V / 32768) equal pieces rounded up to 256 columns (one piece: whole)
+    v_pad = -(-V // 64) * 64
+    if 2 * m_pad * v_pad <= 1 << 30:
+        return v_pad
     n = -(-V // 32768)
     w = -(-(-(-V // n)) // 256) * 256
-    return -(-V // 64) * 64 if w >= V else w
+    return v_pad if w >= V else w
 
 
 def test_pairing_doubles_xm_transpose_and_keeps_dz_for_the_whole_vocabulary(L, bg):
@@ -146,7 +150,7 @@ def test_pairing_doubles_xm_transpose_and_keeps_dz_for_the_whole_vocabulary(L, b
             lean = L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep)))
             pair = L.bgpo_workspace_bytes(ctypes.byref(
                 _prob(bg, B=B, R=R, V=V, H=H, keep_logits=keep, pair_dw=True)))
-            assert pair - lean == 2 * m_pad * H + 2 * (2 * m_pad * v_pad - m_pad * _default_chunk(V))
+            assert pair - lean == 2 * m_pad * H + 2 * (2 * m_pad * v_pad - m_pad * _default_chunk(V, m_pad))
 
 
 def test_vocabulary_chunk_sets_the_dz_buffer(L, bg):
@@ -154,7 +158,7 @@ def test_vocabulary_chunk_sets_the_dz_buffer(L, bg):
     # explicit one, and the whole vocabulary (a chunk of V or more)
     B, R, V, H = 16, 512, 126464, 4096
     m_pad = B * R
-    assert _default_chunk(V) == 31744
+    assert _default_chunk(V, m_pad) == 31744
     size = lambda **kw: L.bgpo_workspace_bytes(ctypes.byref(_prob(bg, B=B, R=R, V=V, H=H, **kw)))
     whole = size(vocab_chunk=1 << 17)
     assert whole - size() == 2 * m_pad * (V - 31744)

@@ -65,9 +65,11 @@ def test_paired_dw_matches_oracle_and_unpaired(bg, name, n_t, keep):
 def test_paired_dw_at_the_full_head(bg):
     """Full LLaDA-8B head (494 vocabulary tiles, K = 4096), 4 samples with few
     masked rows each: the whole dW and dX against the oracle and the unpaired
-    path. The unpaired backward walks the vocabulary in 4 chunks by default,
-    the paired one in 1 (its dZ holds the whole vocabulary): the same dX up to
-    fp32 order; walked in the same chunks, the same dX bits."""
+    path. With so few rows both walk the whole vocabulary at once by default:
+    the same l and dX bits, dW up to fp32 order. Walked in the 4 chunks of
+    31,744 columns that larger batches use by default, paired and unpaired
+    again agree bit for bit in dX, and the chunked dX equals the
+    whole-vocabulary one up to fp32 order."""
     import torch
     from tests.harness import default_vocab_chunk
     wl = CONFIGS["llada8b_r256"].with_(B=2, P=8, R=24, n_t=4, G=2)
@@ -78,14 +80,18 @@ def test_paired_dw_at_the_full_head(bg):
     res = {k: p[k].cpu() for k in ("masks", "ell", "dX", "dW")}
     del p
     a = gpu_run(wl, inp)
-    assert torch.equal(res["ell"], a["ell"].cpu())
-    assert normwise(to64(res["dX"]), to64(a["dX"])) <= VOCAB_ORDER_TOL
+    assert torch.equal(res["ell"], a["ell"].cpu()) and torch.equal(res["dX"], a["dX"].cpu())
     assert normwise(to64(res["dW"]), to64(a["dW"])) <= ORDER_TOL
-    c = gpu_run(wl, inp, pair_dw=True, vocab_chunk=default_vocab_chunk(wl.V))
-    assert bg.get_device_error(c["ws"]) == (0, 0)
-    assert torch.equal(c["ell"], a["ell"]) and torch.equal(c["dX"], a["dX"])
-    assert normwise(to64(c["dW"]), to64(a["dW"])) <= ORDER_TOL
-    del a, c
+    del a
+    chunk = default_vocab_chunk(wl.V)
+    assert chunk == 31744
+    u = gpu_run(wl, inp, vocab_chunk=chunk)
+    c = gpu_run(wl, inp, pair_dw=True, vocab_chunk=chunk)
+    assert bg.get_device_error(u["ws"]) == (0, 0) and bg.get_device_error(c["ws"]) == (0, 0)
+    assert torch.equal(c["ell"], u["ell"]) and torch.equal(c["dX"], u["dX"])
+    assert normwise(to64(c["dW"]), to64(u["dW"])) <= ORDER_TOL
+    assert normwise(to64(u["dX"]), to64(res["dX"])) <= VOCAB_ORDER_TOL
+    del u, c
     torch.cuda.empty_cache()
     o = oracle_run(wl, inp_cpu)
     assert np.array_equal(res["masks"].numpy(), o["masks"])

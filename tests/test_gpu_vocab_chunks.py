@@ -71,14 +71,18 @@ def test_paired_backward_over_the_same_chunks_gives_the_same_dx_bits(bg, name):
 
 
 def test_default_chunks_at_the_full_head(bg):
-    """The LLaDA-8B head (V = 126464) by default runs 4 chunks of 31,744
-    columns; with few masked rows the whole dX and dW against the oracle, and
-    against the whole vocabulary at once."""
+    """The LLaDA-8B head (V = 126464) runs 4 chunks of 31,744 columns by
+    default once the batch's whole-vocabulary dL/dz would exceed 1 GiB (16 x
+    512 responses); here the same chunks on a batch with few masked rows: the
+    whole dX and dW against the oracle, and against the whole vocabulary at
+    once (this batch's default)."""
     import torch
+    from tests.harness import default_vocab_chunk
     wl = CONFIGS["llada8b_r256"].with_(B=2, P=8, R=24, n_t=3, G=2)
+    assert default_vocab_chunk(wl.V, 16 * 512) == 31744 and default_vocab_chunk(wl.V, 48) == 0
     inp_cpu = make_inputs(wl)
     inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
-    c = gpu_run(wl, inp)
+    c = gpu_run(wl, inp, vocab_chunk=31744)
     assert bg.get_device_error(c["ws"]) == (0, 0)
     res = {k: c[k].cpu() for k in ("masks", "ell", "dX", "dW")}
     del c

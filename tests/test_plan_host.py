@@ -182,14 +182,16 @@ def test_forward_regions_fit_the_documented_bound(plan):
 
 def test_vocabulary_chunks(plan):
     # default chunks: V split evenly into ceil(V / 32768) pieces rounded up to
-    # 256 columns (one piece: the whole vocabulary, roundup(V, 64)); with dW
-    # pairing one chunk; dZ holds one chunk unless it must hold them all
+    # 256 columns (one piece: the whole vocabulary, roundup(V, 64)); one chunk
+    # with dW pairing or when the whole vocabulary's dZ fits 1 GiB; dZ holds one
+    # chunk unless it must hold them all
     for L in plan["layout"]:
         V = L["V"]
         v_pad = _ceil(V, 64) * 64
         n = _ceil(V, 32768)
         w = _ceil(_ceil(V, n), 256) * 256
-        vc = v_pad if (L["pair"] or w >= V) else w
+        small = 2 * L["m_pad"] * v_pad <= 1 << 30      # whole-vocabulary dZ within 1 GiB
+        vc = v_pad if (L["pair"] or small or w >= V) else w
         assert L["vc"] == vc and L["n_vc"] == _ceil(V, vc)
         assert (L["n_vc"] - 1) * vc < V <= L["n_vc"] * vc
         last = V - (L["n_vc"] - 1) * vc
