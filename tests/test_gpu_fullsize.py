@@ -9,10 +9,11 @@ error word.
 
 test_full_size_complete_parity compares everything element by element for
 the MC samples with the most masked rows that the fp64 oracle can afford
-inside the GPU test budget: a pair of samples whose dW shares one GEMM
-(BGPO_FLAG_PAIR_DW, as the bench step runs) on both LLaDA-8B workloads, and
-one sample on the Dream-7B workload (each of its samples has 14-18k masked
-rows): every l_b of those samples, all of dX and all of dW.
+inside the GPU test budget: the last pair of samples, whose dW shares one
+GEMM (BGPO_FLAG_PAIR_DW, as the bench step runs), on both LLaDA-8B
+workloads, and one sample on the Dream-7B workload (each of its samples has
+14-18k masked rows, a pair would take the oracle about 5 minutes): every l_b
+of those samples, all of dX and all of dW.
 """
 import numpy as np
 import pytest
@@ -140,9 +141,11 @@ def test_keep_logits_bit_identical_at_full_head(bg):
 
 
 # (workload, first MC sample, dW pairing): the checked samples are j0 (and
-# j0 + 1 when paired); each LLaDA-8B pair has more than 4,400 masked rows per
-# sample, where the operand reused across waves no longer stays in L2
-COMPLETE = [("llada8b_r256", 6, True), ("llada8b_r512_onpolicy", 8, True), ("dream7b", 8, False)]
+# j0 + 1 when paired). On both LLaDA-8B workloads the pair is the last one
+# (n_t - 2, n_t - 1), the most masked rows under stratified t: 7,386 + 7,945 on
+# the bench workload, where the operand reused across waves no longer stays in
+# L2 and one paired dW GEMM runs over K = 7,424 + 7,945 = 15,369 rows
+COMPLETE = [("llada8b_r256", 6, True), ("llada8b_r512_onpolicy", 14, True), ("dream7b", 8, False)]
 
 
 @pytest.mark.parametrize("name,j0,pair", COMPLETE)
