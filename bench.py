@@ -54,8 +54,8 @@ UNIT = "tokens/s"
 # reports traffic as null); the dX and dW GEMMs' traffic is not proportional to
 # their tiles and is not estimated.
 TRAFFIC = {
-    "sha": "f6588a6ec6612107068d29bdc644ed9d2fdede82593cf02d4c8a8cc593940d71",
-    "bytes_per_tile": {"lmhead_fwd_lse": 1.67e5, "lmhead_dz": 3.41e5},
+    "sha": "a9b2152e2f17e6083ace0813fa5e7f3a8aa3d2120560f4319f4ac99c9f75dcf9",
+    "bytes_per_tile": {"lmhead_fwd_lse": 1.68e5, "lmhead_dz": 3.35e5},
     "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by pair tiles",
 }
 
