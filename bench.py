@@ -294,9 +294,11 @@ def main():
         # NCCL's own start-up lines (ranks, devices) stay in the log
         os.environ.setdefault("NCCL_DEBUG", "INFO")
         os.environ.setdefault("NCCL_DEBUG_SUBSYS", "INIT")
-        dist.init_process_group("nccl")
+    # each rank drives the GPU of its local rank; select it before NCCL binds
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
 
     import paper_2510_11683_gb300 as bg
     from paper_2510_11683_gb300 import build as B
