@@ -97,6 +97,16 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   return mbar_wait_timeout(bar, parity, abort, kWaitTimeoutNs);
 }
 
+// 2^x by the special-function unit's approximation (PTX ex2.approx.ftz.f32:
+// relative error within 2^-22, subnormal inputs and results flushed to zero).
+// The arguments here are logits minus their row's log-sum-exp or running
+// maximum, so a flushed result is below 2^-126 of the row's largest term.
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // ---- TMA -----------------------------------------------------------------------
 
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {

@@ -304,20 +304,34 @@ __device__ __forceinline__ void epi_fwd(const GemmParams& p, const CUtensorMap* 
     tmem_ld_32x32b_x32(tb + c * 32, raw);
     tmem_ld_wait();
     const int nvalid = min(32, V - col0);
-    float cm = -INFINITY;
+    // the row's target lies in this sub-tile for about one sub-tile in 4000:
+    // test it once instead of once per column
+    if ((uint32_t)(y - col0) < 32u) {
 #pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const float z = bits_f(raw[k]);
-      if (k < nvalid) cm = fmaxf(cm, z);
-      if (col0 + k == y) { tl = z; hit = true; }
+      for (int k = 0; k < 32; ++k)
+        if (col0 + k == y) { tl = bits_f(raw[k]); hit = true; }
     }
-    const float mn = fmaxf(m, cm);
-    const float mnl = mn * kLog2e;
+    float cm = -INFINITY;
     float acc = 0.f;
+    float mn;
+    if (nvalid == 32) {  // warp-uniform: every column lies inside the vocabulary
 #pragma unroll
-    for (int k = 0; k < 32; ++k)
-      if (k < nvalid) acc += exp2f(fmaf(bits_f(raw[k]), kLog2e, -mnl));
-    s = s * exp2f((m - mn) * kLog2e) + acc;
+      for (int k = 0; k < 32; ++k) cm = fmaxf(cm, bits_f(raw[k]));
+      mn = fmaxf(m, cm);
+      const float mnl = mn * kLog2e;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) acc += ex2_ftz(fmaf(bits_f(raw[k]), kLog2e, -mnl));
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < nvalid) cm = fmaxf(cm, bits_f(raw[k]));
+      mn = fmaxf(m, cm);
+      const float mnl = mn * kLog2e;
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < nvalid) acc += ex2_ftz(fmaf(bits_f(raw[k]), kLog2e, -mnl));
+    }
+    s = s * ex2_ftz((m - mn) * kLog2e) + acc;
     m = mn;
     if (p.w.zc != nullptr) {  // kernel-uniform; col0 < V <= v_pad, both multiples of 32
       uint4 chunk[8];
@@ -356,10 +370,15 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
   const int32_t v0 = (int32_t)p.v_begin + t.n_blk * kBN;
   const int32_t V = (int32_t)p.g.V;
   const int32_t shift = (int32_t)(p.dz_col0 - p.v_begin);   // vocabulary entry -> dZ column
+  const float nw = -w;
 #pragma unroll 1
   for (int c = 0; c < kBN / 64; ++c) {
     const int32_t col0 = v0 + c * 64;
     if (col0 + shift >= p.w.dz_cols) break;  // warp-uniform
+    // almost every sub-tile of a row lies inside the vocabulary and away from
+    // the row's target: there dz = -w e^{z - lse}, the same value the general
+    // expression gives (w (0 - p) = (-w) p exactly)
+    const bool plain = valid && col0 + 64 <= V && (uint32_t)(y - col0) >= 64u;
     uint4 chunk[8];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -367,17 +386,26 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
       tmem_ld_32x32b_x32(tb + c * 64 + h * 32, raw);
       tmem_ld_wait();
       uint32_t packed[16];
+      if (plain) {
 #pragma unroll
-      for (int k = 0; k < 32; k += 2) {
-        float d[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int32_t col = col0 + h * 32 + k + e;
-          const float pr = exp2f(fmaf(bits_f(raw[k + e]), kLog2e, -lse_l2));
-          const float v = w * ((col == y ? 1.f : 0.f) - pr);
-          d[e] = (valid && col < V) ? v : 0.f;
+        for (int k = 0; k < 32; k += 2) {
+          const float d0 = nw * ex2_ftz(fmaf(bits_f(raw[k]), kLog2e, -lse_l2));
+          const float d1 = nw * ex2_ftz(fmaf(bits_f(raw[k + 1]), kLog2e, -lse_l2));
+          packed[k / 2] = pack_bf16x2(d0, d1);
         }
-        packed[k / 2] = pack_bf16x2(d[0], d[1]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float d[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int32_t col = col0 + h * 32 + k + e;
+            const float pr = ex2_ftz(fmaf(bits_f(raw[k + e]), kLog2e, -lse_l2));
+            const float v = w * ((col == y ? 1.f : 0.f) - pr);
+            d[e] = (valid && col < V) ? v : 0.f;
+          }
+          packed[k / 2] = pack_bf16x2(d[0], d[1]);
+        }
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q)

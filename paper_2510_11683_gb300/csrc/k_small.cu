@@ -321,7 +321,7 @@ __global__ void __launch_bounds__(kDzThreads, 4)
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int32_t col = (int32_t)(v_begin + v * 8) + e + h;
-          const float pr = exp2f(fmaf(zz[e + h], kLog2e, -lse_l2));
+          const float pr = ex2_ftz(fmaf(zz[e + h], kLog2e, -lse_l2));
           const float val = wr * ((col == y ? 1.f : 0.f) - pr);
           d[h] = (valid && col < V) ? val : 0.f;
         }
