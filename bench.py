@@ -46,17 +46,19 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum of the forward and dZ GEMMs per
-# 256 x 256 pair tile, from ncu captures of single launches on the small case
-# llada8b_r512_b8 (MC samples 12 and 13, 13 and 14 row blocks x 494 vocabulary
-# tiles, dW paired as in the bench step); a launch's traffic is scaled by its
-# pair tiles. Valid while the GEMM sources hash to `sha` (otherwise the line
-# reports traffic as null); the dX and dW GEMMs' traffic is not proportional to
-# their tiles and is not estimated.
+# dram__bytes_read.sum + dram__bytes_write.sum per unit of work, from ncu
+# captures of single launches on the small case llada8b_r512_b8 (MC samples 12
+# and 13, 13 and 14 row blocks, dW paired as in the bench step): per 256 x 256
+# pair tile for the forward and dZ GEMMs (K = H), per pair tile and 64-column
+# K block for the dX GEMM (K = the vocabulary, split or not). A bench launch's
+# traffic is that figure times its units. Valid while the GEMM sources hash to
+# `sha` (otherwise the line reports traffic as null); the paired dW GEMM's
+# traffic is not proportional to its units and is not estimated.
 TRAFFIC = {
-    "sha": "a9b2152e2f17e6083ace0813fa5e7f3a8aa3d2120560f4319f4ac99c9f75dcf9",
-    "bytes_per_tile": {"lmhead_fwd_lse": 1.68e5, "lmhead_dz": 3.35e5},
-    "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by pair tiles",
+    "sha": "b09fe802cf16f4b1a53e8110949a5cacfcfd7b4efa625a9cef3bd6e203b4d2cc",
+    "bytes_per_tile": {"lmhead_fwd_lse": 1.82e5, "lmhead_dz": 3.49e5},
+    "bytes_per_tile_kblock": {"dx_gemm": 1.35e4},
+    "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by units",
 }
 
 
@@ -409,11 +411,13 @@ def main():
         dom_avg_s = dom_ms / dom_launches / 1e3
         achieved = dom_flops_per_launch / dom_avg_s / 1e12
         traffic = None
-        per_tile = TRAFFIC["bytes_per_tile"].get(dom)
-        if headline_mode and per_tile and TRAFFIC["sha"] == kernel_sha():
-            # pair tiles per launch: row blocks of each sample x vocabulary tiles
-            tiles = sum(-(-m // 256) for m in rows_per_sample) * (-(-V // 256)) / n_t
-            traffic = per_tile * tiles
+        if headline_mode and TRAFFIC["sha"] == kernel_sha():
+            row_blocks = sum(-(-m // 256) for m in rows_per_sample) / n_t   # per launch
+            if dom in TRAFFIC["bytes_per_tile"]:
+                traffic = TRAFFIC["bytes_per_tile"][dom] * row_blocks * (-(-V // 256))
+            elif dom in TRAFFIC["bytes_per_tile_kblock"]:
+                traffic = (TRAFFIC["bytes_per_tile_kblock"][dom] * row_blocks * (-(-H // 256))
+                           * (-(-V // 64)))
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "traffic_source": TRAFFIC["source"] if traffic is not None else None,
