@@ -540,13 +540,15 @@ def main():
 
 def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0,
             barrier=lambda: None, pair=False):
-    from paper_2510_11683_gb300.dp import allreduce_dw
     """Same step through host buffers: every step copies its inputs (X, W, Y,
-    rewards or A, l_old) from pinned host memory and reads its results (l and g)
-    back. Copies run on a second stream into the other of two device buffer
-    sets, so step k+1's inputs travel while step k computes; all copies lie
-    inside the timed region."""
+    rewards or A, l_old) from pinned host memory and copies its results (l and
+    g) back to pinned host memory, where the host reads them. Input copies run
+    on a second stream into the other of two device buffer sets, so step k+1's
+    inputs travel while step k computes; the host reads step k - 1's results
+    while step k runs, as a training loop that logs the previous step's loss
+    does. All copies and reads lie inside the timed region."""
     import torch
+    from paper_2510_11683_gb300.dp import allreduce_dw
     n_t, Bsz = wl.n_t, wl.B
     host = {
         "X": inp_cpu["X"].pin_memory(), "W": inp_cpu["W"].pin_memory(),
@@ -555,8 +557,8 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     adv_key = "A" if inp_cpu["A"] is not None else "rewards"
     host["adv"] = inp_cpu[adv_key].pin_memory()
     bufs = [{k: torch.empty_like(v, device=dev) for k, v in host.items()} for _ in range(2)]
-    out_ell = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
-    out_g = torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory()
+    out_ell = [torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory() for _ in range(2)]
+    out_g = [torch.empty((n_t, Bsz), dtype=torch.float32).pin_memory() for _ in range(2)]
     prob = bg.problem_from(wl, b_offset=b_offset, pair_dw=pair)
     ws = bg.alloc_workspace(prob, dev)
     A = torch.empty(Bsz, dtype=torch.float32, device=dev)
@@ -566,11 +568,13 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     dX = torch.zeros((Bsz, wl.R, wl.H), dtype=torch.float32, device=dev)
     dW = torch.zeros((wl.V, wl.H), dtype=torch.float32, device=dev)
     h2d = sum(v.numel() * v.element_size() for v in host.values())
-    d2h = out_ell.numel() * 4 + out_g.numel() * 4
+    d2h = out_ell[0].numel() * 4 + out_g[0].numel() * 4
     compute = torch.cuda.current_stream()
     copy = torch.cuda.Stream(device=dev)
     copied = [torch.cuda.Event(), torch.cuda.Event()]
     consumed = [torch.cuda.Event(), torch.cuda.Event()]
+    ready = [torch.cuda.Event(), torch.cuda.Event()]   # a step's results are on the host
+    seen = []                                          # what the host read, per step
 
     def issue_copy(k):
         slot = k % 2
@@ -595,8 +599,13 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
             bg.elbo_bwd_accumulate(prob, j, b["X"], b["W"], b["Y"], coef[j], ws, dX, dW)
         allreduce_dw(dW)          # the data-parallel exchange (a no-op on one rank)
         consumed[slot].record(compute)
-        out_ell.copy_(ell, non_blocking=True)
-        out_g.copy_(g, non_blocking=True)
+        out_ell[slot].copy_(ell, non_blocking=True)
+        out_g[slot].copy_(g, non_blocking=True)
+        ready[slot].record(compute)
+
+    def read(k):
+        ready[k % 2].synchronize()
+        seen.append((float(out_ell[k % 2].sum()), float(out_g[k % 2].sum())))
 
     def run(steps):
         issue_copy(0)
@@ -604,7 +613,9 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
             if k + 1 < steps:
                 issue_copy(k + 1)
             compute_step(k)
-            torch.cuda.current_stream().synchronize()   # the step's results are on the host
+            if k > 0:
+                read(k - 1)          # step k - 1's results, while step k runs
+        read(steps - 1)
     for e in consumed:
         e.record(compute)
     run(max(1, min(args.warmup, 2)))
@@ -618,7 +629,9 @@ def e2e_leg(bg, wl, inp_cpu, ell_old_cpu, masked_per_step, args, dev, b_offset=0
     barrier()
     return {"value": masked_per_step / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps,
-            "pipelining": "inputs of step k+1 copied on a second stream during step k"}
+            "pipelining": "inputs of step k+1 copied on a second stream during step k; the host "
+                          "reads step k-1's results during step k",
+            "results_finite": bool(all(np.isfinite(v) for pair in seen for v in pair))}
 
 
 def run_profile_sample(args, wl):
