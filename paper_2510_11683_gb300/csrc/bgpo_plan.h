@@ -24,6 +24,18 @@ constexpr int kBNHalf = 128;     // B columns staged by each CTA of the pair
 constexpr int kBK = 64;          // K per pipeline stage: one 128-byte swizzle row of bf16
 constexpr int kUmmaK = 16;       // K of one tcgen05.mma kind::f16 instruction
 constexpr int kStages = 6;       // TMA -> MMA pipeline depth
+// The dX GEMM's tiles are kDxWide accumulators wide (256 x 512 for 2): each
+// K block of A then feeds kDxWide MMAs, so the operand stream per flop into
+// shared memory is 3/4 of a 256 x 256 tile's, and a wave of tiles covers all
+// of H with half as many W column blocks re-read per row block. Both of the
+// pair's 256-column accumulators hold one tile (the epilogue does not overlap
+// the next tile's main loop), with kDxStages stages of 48 KB per CTA.
+#ifndef BGPO_DX_WIDE
+#define BGPO_DX_WIDE 2
+#endif
+constexpr int kDxWide = BGPO_DX_WIDE;
+static_assert(kDxWide == 1 || kDxWide == 2, "dX tile width: one or two accumulators");
+constexpr int kDxStages = kDxWide == 2 ? 4 : kStages;
 constexpr int kMaxSplits = 16;   // split-K limit of the dX GEMM
 // Widest vocabulary chunk of the backward by default: dZ is formed, used by
 // the dX GEMM and the dW GEMM one chunk of at most this many columns at a
@@ -64,6 +76,9 @@ enum KernelId : int32_t {
 
 BGPO_HD int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 BGPO_HD int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
+
+// Column tiles of the dX GEMM for `tiles_h` hidden-size blocks of kBN columns.
+BGPO_HD int64_t dx_tiles_n(int64_t tiles_h) { return ceil_div(tiles_h, kDxWide); }
 
 // Split-K count of the dX GEMM (K = vocabulary) for `mb` pair row blocks times
 // `tiles_n` column tiles on `num_pairs` CTA pairs: the smallest s whose
@@ -178,13 +193,15 @@ struct WsLayout {
 BGPO_HD size_t align_ws(size_t x) { return (x + 1023) & ~(size_t)1023; }
 
 // Pair row blocks (256 rows) the split-K partial buffer holds, which bounds the
-// splits s of a sample with mb row blocks to s * mb <= cap: two splits at the
+// splits s of a sample with mb row blocks to s * mb <= cap: three splits at the
 // largest mb, up to kMaxSplits for small mb (measured: a second split takes
-// 6-8% off a dX GEMM whose unsplit tiles leave a last wave 20% full).
+// 6-8% off a dX GEMM whose unsplit tiles leave a last wave 20% full; with
+// 256 x 512 tiles, room for a third split took 1.5% off the dX GEMMs of a
+// step against room for two).
 BGPO_HD int64_t dxp_row_block_cap(const Geometry& g) {
   const int64_t mb_max = g.m_pad / kPairM;
   const int64_t small = 4 * mb_max < 4 * kMaxSplits ? 4 * mb_max : 4 * kMaxSplits;
-  int64_t cap = 2 * mb_max > small ? 2 * mb_max : small;
+  int64_t cap = 3 * mb_max > small ? 3 * mb_max : small;
   return cap > kMaxSplits ? cap : kMaxSplits;
 }
 

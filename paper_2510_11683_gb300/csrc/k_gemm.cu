@@ -4,17 +4,20 @@
 // CTA pair computes 256 x 256 fp32 tiles with tcgen05.mma.cta_group::2: CTA r
 // of the pair stages rows [128 r, 128 r + 128) of the A tile and columns
 // [128 r, 128 r + 128) of the B tile, and holds accumulator rows
-// [128 r, 128 r + 128) in its TMEM. Roles in each CTA (192 threads):
+// [128 r, 128 r + 128) in its TMEM. The dX GEMM's tiles are kDxWide such
+// tiles side by side, sharing their A tile. Roles in each CTA (192 threads):
 //   warp 0      TMA producer: 128-byte-swizzled bf16 boxes into a 6-stage ring
-//               of 32 KB; every copy of both CTAs completes on the even CTA's
+//               of 32 KB (dX: 4 stages of 48 KB); every copy of both CTAs completes on the even CTA's
 //               "full" barrier, which the even CTA alone arms with both CTAs'
 //               transaction bytes (a negative transaction count in between is
 //               allowed)
 //   warp 1      TMEM allocation (pair, 512 columns = two accumulators); in the
-//               even CTA also the MMA issuer (M = 256, N = 256, K = 16)
+//               even CTA also the MMA issuer (M = 256, N = 256, K = 16; the
+//               dX GEMM issues one per accumulator of its tile)
 //   warps 2-5   epilogue: tcgen05.ld of this CTA's accumulator rows, fused
 //               per-kind epilogue, TMA stores / reductions from shared memory
-// The epilogue of tile n overlaps the main loop of tile n+1.
+// The epilogue of tile n overlaps the main loop of tile n+1, except in the dX
+// GEMM when its tiles occupy both accumulators.
 //
 // Kinds (Xm = gathered masked hidden states [M, H], W = LM head [V, H]):
 //   GEMM_FWD  z = Xm W^T; epilogue: online max / sum-exp per (row, vocab tile)
@@ -25,7 +28,7 @@
 //             vocabulary chunk of the backward; epilogue: dz = w_r (onehot -
 //             e^{z - lse}) stored as bf16 (gradient of Eq. 4 weighted by
 //             Eq. 13's dL/dl).
-//   GEMM_DX   dXm += dZ_c W_c (K = the chunk's vocabulary): split-K partials in
+//   GEMM_DX   dXm += dZ_c W_c (K = the chunk's vocabulary; 256 x 512 tiles): split-K partials in
 //             fp32, stored by the first chunk and added by the later ones, or,
 //             when the launch needs no split, added straight into the dX rows.
 //   GEMM_DW   dW[chunk rows] += dZ_c^T Xm (K = masked rows; Xm read as its
@@ -93,7 +96,7 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_
     w.units = w.tiles_m * w.tiles_n;
   } else if (KIND == GEMM_DX) {
     w.tiles_m = ceil_div(M, kPairM);
-    w.tiles_n = p.g.tiles_h;
+    w.tiles_n = dx_tiles_n(p.g.tiles_h);
     w.kb_total = ceil_div(p.v_end - p.v_begin, kBK);
     // one split count for every chunk of the sample (the partials of split s
     // accumulate over the chunks), bounded by the narrowest chunk's K blocks
@@ -147,10 +150,19 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
 // staging buffers (the forward GEMM stages its fp32 logits there when it keeps
 // them).
 template <int KIND>
+struct Shape {
+  static constexpr int nacc = KIND == GEMM_DX ? kDxWide : 1;  // accumulators per tile
+  static constexpr int bufs = 2 / nacc;                        // tiles in TMEM at once
+  static constexpr int stages = KIND == GEMM_DX ? kDxStages : kStages;
+  static constexpr uint32_t b_bytes = nacc * kTileBBytes;      // B bytes per CTA and stage
+};
+
+template <int KIND>
 struct SmemPlan {
-  static constexpr int stages = kStages;
+  static constexpr int stages = Shape<KIND>::stages;
   static constexpr uint32_t epi_bytes = kEpiBytes;
-  static constexpr uint32_t bytes = stages * kStageBytes + epi_bytes + 1024 + 1024;
+  static constexpr uint32_t bytes =
+      stages * (kTileABytes + Shape<KIND>::b_bytes) + epi_bytes + 1024 + 1024;
   static_assert(bytes <= 232448, "shared memory per CTA");
 };
 
@@ -181,7 +193,8 @@ __device__ __forceinline__ int64_t b_base(const GemmParams& p) {
 template <int KIND>
 __device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit& t, uint32_t rank) {
   const int64_t a0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM;
-  const int64_t b0 = b_base<KIND>(p) + (int64_t)t.n_blk * kBN + (int64_t)rank * kBNHalf;
+  const int64_t b0 =
+      b_base<KIND>(p) + (int64_t)t.n_blk * Shape<KIND>::nacc * kBN + (int64_t)rank * kBNHalf;
   uint32_t bytes = 0;
   if (!Majors<KIND>::a_mn) {
     bytes += kTileABytes;
@@ -193,8 +206,9 @@ __device__ __forceinline__ uint32_t stage_bytes(const GemmParams& p, const Unit&
   if (!Majors<KIND>::b_mn) {
     if (b0 < b_rows<KIND>(p)) bytes += kTileBBytes;
   } else {
-    for (int c = 0; c < kBNHalf / 64; ++c)
-      if (b0 + c * 64 < p.g.H) bytes += kMnChunkBytes;
+    for (int g = 0; g < Shape<KIND>::nacc; ++g)
+      for (int c = 0; c < kBNHalf / 64; ++c)
+        if (b0 + g * kBN + c * 64 < p.g.H) bytes += kMnChunkBytes;
   }
   return bytes;
 }
@@ -210,7 +224,8 @@ __device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMa
                                            uint32_t rank, int64_t roff) {
   const int32_t a0 =
       t.m_blk * kPairM + (int32_t)rank * kBM + (KIND == GEMM_DX ? (int32_t)roff : 0);
-  const int64_t b0 = b_base<KIND>(p) + (int64_t)t.n_blk * kBN + (int64_t)rank * kBNHalf;
+  const int64_t b0 =
+      b_base<KIND>(p) + (int64_t)t.n_blk * Shape<KIND>::nacc * kBN + (int64_t)rank * kBNHalf;
   if (!Majors<KIND>::a_mn) {
     const int32_t ka = kb * kBK + (KIND == GEMM_DX ? (int32_t)p.dz_col0 : 0);
     tma_load_2d_pair(sa, ma, cbar, ka, a0);
@@ -226,12 +241,16 @@ __device__ __forceinline__ void load_stage(const GemmParams& p, const CUtensorMa
   if (!Majors<KIND>::b_mn) {
     if (b0 < b_rows<KIND>(p)) tma_load_2d_pair(sb, mb, cbar, kb * kBK, (int32_t)b0);
   } else {
-    // W columns of this CTA (GEMM_DX): 2 boxes of 64 x 64, rows from the chunk's start
+    // W columns of this CTA (GEMM_DX): 2 boxes of 64 x 64 per accumulator of the
+    // tile (accumulator g's at sb + g * kTileBBytes), rows from the chunk's start
     const int32_t kw = (int32_t)(p.v_begin + (int64_t)kb * kBK);
 #pragma unroll
-    for (int c = 0; c < kBNHalf / 64; ++c)
-      if (b0 + c * 64 < p.g.H)
-        tma_load_2d_pair(sb + c * kMnChunkBytes, mb, cbar, (int32_t)b0 + c * 64, kw);
+    for (int g = 0; g < Shape<KIND>::nacc; ++g)
+#pragma unroll
+      for (int c = 0; c < kBNHalf / 64; ++c)
+        if (b0 + g * kBN + c * 64 < p.g.H)
+          tma_load_2d_pair(sb + g * kTileBBytes + c * kMnChunkBytes, mb, cbar,
+                           (int32_t)(b0 + g * kBN + c * 64), kw);
   }
 }
 
@@ -425,53 +444,64 @@ __device__ __forceinline__ void epi_dz(const GemmParams& p, const CUtensorMap* m
 // writer per launch and the chunks run in order, so the sum is deterministic;
 // rows >= M hold zeros). Without split-K every dX element has exactly this one
 // contribution in the launch, so the lane adds its row's sub-tile straight
-// into dX[b, i] (the row the compaction recorded), 128 contiguous bytes per
-// sub-tile, and the split reduction after the last chunk has nothing to do.
+// into dX[b, i] (the row the compaction recorded) with 16-byte atomic adds,
+// which need no round trip: each element still receives one addition, and the
+// split reduction after the last chunk has nothing to do.
+__device__ __forceinline__ void dx_sub(const GemmParams& p, const CUtensorMap* map_c,
+                                       const Work& wk, float4* drow, int32_t h0, int32_t prow0,
+                                       int c, const uint32_t (&raw)[32], int lane, EpiStage& st) {
+  if (wk.splits == 1) {  // launch-uniform
+    if (drow) {
+      // 16-byte pieces of this sub-tile inside the row (H is a multiple of 8)
+      const int nq = min(8, ((int32_t)p.g.H - (h0 + c * 32)) / 4);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (q >= nq) break;
+        atomicAdd(drow + c * 8 + q, make_float4(bits_f(raw[4 * q]), bits_f(raw[4 * q + 1]),
+                                                bits_f(raw[4 * q + 2]), bits_f(raw[4 * q + 3])));
+      }
+    }
+    return;
+  }
+  uint4 chunk[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
+  const uint32_t sbuf = st.acquire(lane);
+  stage_row(sbuf, lane, chunk);
+  if (p.chunk == 0)
+    st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, h0 + c * 32, prow0); });
+  else
+    st.release(lane, sbuf, [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, prow0); });
+}
+
+// `nb`: the 256-column block of dX this accumulator holds. The TMEM load of
+// sub-tile c + 1 is in flight while sub-tile c is written out.
 __device__ __forceinline__ void epi_dx(const GemmParams& p, const CUtensorMap* map_c, int32_t M,
-                                       const Work& wk, const Unit& t, int64_t row0, int lane,
-                                       uint32_t tb, EpiStage& st) {
-  const int32_t h0 = t.n_blk * kBN;
+                                       const Work& wk, const Unit& t, int32_t nb, int64_t row0,
+                                       int lane, uint32_t tb, EpiStage& st) {
+  const int32_t h0 = nb * kBN;
+  const int32_t nsub = min(kBN / 32, ((int32_t)p.g.H - h0 + 31) / 32);  // inside H
+  if (nsub <= 0) return;  // a column block past H (warp-uniform)
   const int32_t prow0 = (int32_t)(t.split * wk.tiles_m * kPairM + row0);
   const int64_t r = row0 + lane;
   float4* drow = nullptr;
-  const int32_t H = (int32_t)p.g.H;
   if (wk.splits == 1 && r < M &&
       BGPO_IN_BOUNDS(p.w.err, p.w.rows[r] >= 0 && p.w.rows[r] < p.g.m_cap, KID_DX_GEMM * 16 + 10))
     drow = reinterpret_cast<float4*>(p.dX + (int64_t)p.w.rows[r] * p.g.H + h0);
+  uint32_t ra[32], rb[32];
+  tmem_ld_32x32b_x32(tb, ra);
+  tmem_ld_wait_regs(ra);
 #pragma unroll 1
-  for (int c = 0; c < kBN / 32; ++c) {
-    if (h0 + c * 32 >= p.g.H) break;  // warp-uniform
-    uint32_t raw[32];
-    tmem_ld_32x32b_x32(tb + c * 32, raw);
-    tmem_ld_wait();
-    if (wk.splits == 1) {  // launch-uniform
-      if (drow) {
-        // 16-byte pieces of this sub-tile inside the row (H is a multiple of 8)
-        const int nq = min(8, (H - (h0 + c * 32)) / 4);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          if (q >= nq) break;
-          float4 o = drow[c * 8 + q];
-          o.x += bits_f(raw[4 * q]);
-          o.y += bits_f(raw[4 * q + 1]);
-          o.z += bits_f(raw[4 * q + 2]);
-          o.w += bits_f(raw[4 * q + 3]);
-          drow[c * 8 + q] = o;
-        }
-      }
-      continue;
+  for (int c = 0; c < nsub; c += 2) {
+    if (c + 1 < nsub) tmem_ld_32x32b_x32(tb + (uint32_t)(c + 1) * 32, rb);
+    dx_sub(p, map_c, wk, drow, h0, prow0, c, ra, lane, st);
+    if (c + 1 < nsub) {
+      tmem_ld_wait_regs(rb);
+      if (c + 2 < nsub) tmem_ld_32x32b_x32(tb + (uint32_t)(c + 2) * 32, ra);
+      dx_sub(p, map_c, wk, drow, h0, prow0, c + 1, rb, lane, st);
+      if (c + 2 < nsub) tmem_ld_wait_regs(ra);
     }
-    uint4 chunk[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q)
-      chunk[q] = make_uint4(raw[4 * q], raw[4 * q + 1], raw[4 * q + 2], raw[4 * q + 3]);
-    const uint32_t sbuf = st.acquire(lane);
-    stage_row(sbuf, lane, chunk);
-    if (p.chunk == 0)
-      st.release(lane, sbuf, [&](uint32_t a) { tma_store_2d(map_c, a, h0 + c * 32, prow0); });
-    else
-      st.release(lane, sbuf,
-                 [&](uint32_t a) { tma_reduce_add_2d(map_c, a, h0 + c * 32, prow0); });
   }
 }
 
@@ -523,9 +553,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+  constexpr uint32_t kBBytes = Shape<KIND>::b_bytes;
+  constexpr int kNacc = Shape<KIND>::nacc;
+  constexpr int kBufs = Shape<KIND>::bufs;
   uint8_t* s_a = smem;
   uint8_t* s_b = smem + kSt * kTileABytes;
-  uint8_t* s_epi = s_b + kSt * kTileBBytes;   // 4 warps x 2 staging buffers
+  uint8_t* s_epi = s_b + kSt * kBBytes;   // 4 warps x 2 staging buffers
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_epi + SmemPlan<KIND>::epi_bytes);
   uint64_t* full = bars;                      // [kSt] TMA (both CTAs) -> MMA; even CTA's
   uint64_t* empty = bars + kSt;           // [kSt] MMA -> TMA of each CTA
@@ -615,7 +648,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t cbar = map_to_cta(smem_addr(&full[stage]), 0);
           if (rank == 0) mbar_arrive_expect_tx(smem_addr(&full[stage]), bytes);
           load_stage<KIND>(p, &map_a, &map_b, smem_addr(s_a + stage * kTileABytes),
-                           smem_addr(s_b + stage * kTileBBytes), cbar, t, kb, rank, roff);
+                           smem_addr(s_b + stage * kBBytes), cbar, t, kb, rank, roff);
           issued = true;
           if (++stage == kSt) { stage = 0; phase ^= 1u; }
         }
@@ -643,8 +676,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int it = 0;
       for (int64_t u = pair; u < wk.units && ok; u += num_pairs, ++it) {
         const Unit t = unit_of<KIND>(wk, u);
-        const int acc = it & 1;
-        const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+        const int acc = it % kBufs;
+        const uint32_t acc_phase = (uint32_t)(it / kBufs) & 1u;
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
@@ -652,14 +685,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (!mbar_wait(smem_addr(&full[stage]), phase, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sa = smem_addr(s_a + stage * kTileABytes);
-          const uint32_t sb = smem_addr(s_b + stage * kTileBBytes);
+          const uint32_t sb = smem_addr(s_b + stage * kBBytes);
 #pragma unroll
           for (int k = 0; k < kBK / kUmmaK; ++k) {
             const uint64_t ad = Majors<KIND>::a_mn ? smem_desc_sw128(sa + k * 2048, kMnChunkBytes, 1024)
                                                    : smem_desc_sw128(sa + k * 32, 16, 1024);
-            const uint64_t bd = Majors<KIND>::b_mn ? smem_desc_sw128(sb + k * 2048, kMnChunkBytes, 1024)
-                                                   : smem_desc_sw128(sb + k * 32, 16, 1024);
-            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+            for (int g = 0; g < kNacc; ++g) {
+              const uint32_t sbg = sb + (uint32_t)g * kTileBBytes;
+              const uint64_t bd = Majors<KIND>::b_mn
+                                      ? smem_desc_sw128(sbg + k * 2048, kMnChunkBytes, 1024)
+                                      : smem_desc_sw128(sbg + k * 32, 16, 1024);
+              umma_bf16_pair(d_tmem + (uint32_t)(g * kBN), ad, bd, idesc,
+                             (kb > 0 || k > 0) ? 1u : 0u);
+            }
           }
           issued = true;
           // frees this stage in both CTAs once these MMAs have read it
@@ -689,8 +728,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int64_t u = pair; u < wk.units; u += num_pairs, ++it) {
       const Unit t = unit_of<KIND>(wk, u);
-      const int acc = it & 1;
-      const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+      const int acc = it % kBufs;
+      const uint32_t acc_phase = (uint32_t)(it / kBufs) & 1u;
       const bool got = mbar_wait(smem_addr(&tfull[acc]), acc_phase, abort_flag);
       if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
       tc_fence_after();
@@ -698,7 +737,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int64_t row0 = (int64_t)t.m_blk * kPairM + (int64_t)rank * kBM + quarter * 32;
       if (KIND == GEMM_FWD) epi_fwd(p, &map_c, M, t, row0, lane, tb, st);
       else if (KIND == GEMM_DZ) epi_dz(p, &map_c, M, t, row0, roff, lane, tb, st);
-      else if (KIND == GEMM_DX) epi_dx(p, &map_c, M, wk, t, row0, lane, tb, st);
+      else if (KIND == GEMM_DX) {
+#pragma unroll 1
+        for (int g = 0; g < kNacc; ++g)
+          epi_dx(p, &map_c, M, wk, t, t.n_blk * kNacc + g, row0, lane, tb + (uint32_t)(g * kBN), st);
+      }
       else epi_dw(p, &map_c, t, row0, lane, tb, st);
       tc_fence_before();
       __syncwarp();

@@ -44,10 +44,11 @@ static void layout(int64_t B, int64_t R, int64_t H, int64_t V) {
   const int64_t cap = dxp_row_block_cap(g);
   for (int64_t mb = 1; mb <= g.m_pad / kPairM; ++mb)
     for (int pairs : {1, 7, 76}) {
-      const int s = dx_splits(mb, g.tiles_h, pairs, g.kb_v, cap);
+      const int s = dx_splits(mb, dx_tiles_n(g.tiles_h), pairs, g.kb_v, cap);
       printf("{\"kind\": \"split\", \"mb\": %lld, \"tiles_n\": %lld, \"pairs\": %d, \"kb\": %lld, "
-             "\"cap\": %lld, \"s\": %d}\n",
-             (long long)mb, (long long)g.tiles_h, pairs, (long long)g.kb_v, (long long)cap, s);
+             "\"cap\": %lld, \"s\": %d, \"tiles_h\": %lld}\n",
+             (long long)mb, (long long)dx_tiles_n(g.tiles_h), pairs, (long long)g.kb_v,
+             (long long)cap, s, (long long)g.tiles_h);
     }
   for (int pair = 0; pair < 2; ++pair) {
     const WsLayout L = make_ws_layout(g, false, pair);
@@ -134,6 +135,8 @@ def test_regions_up_to_xm_do_not_move_with_the_flags(plan):
 def test_dx_split_choice(plan):
     for r in plan["split"]:
         mb, tn, pairs, kb, cap, s = r["mb"], r["tiles_n"], r["pairs"], r["kb"], r["cap"], r["s"]
+        # dX tiles are 256 x 512: two 256-column blocks of H each
+        assert tn == _ceil(r["tiles_h"], 2), r
         smax = max(1, min(16, kb, cap // mb))
         assert 1 <= s <= smax, r
         assert s == 1 or s * mb <= cap, r
@@ -145,10 +148,10 @@ def test_dx_split_choice(plan):
             assert all(t(k) > 1.08 * ideal for k in range(1, s)), r
 
 
-def test_split_room_allows_two_splits_at_the_largest_row_count(plan):
+def test_split_room_allows_three_splits_at_the_largest_row_count(plan):
     for L in plan["layout"]:
         mb_max = _ceil(L["B"] * L["R"], 256)
-        assert L["cap"] >= max(2 * mb_max, 16)
+        assert L["cap"] >= max(3 * mb_max, 16)
 
 
 def test_pairing_offsets_are_clamped(plan):
