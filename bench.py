@@ -46,19 +46,19 @@ WORKLOAD = "llada8b_r512_onpolicy"
 METRIC = "masked tokens/s (fwd+bwd)"
 UNIT = "tokens/s"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per unit of work, from ncu
-# captures of single launches on the small case llada8b_r512_b8 (MC samples 12
-# and 13, 13 and 14 row blocks, dW paired as in the bench step): per 256 x 256
-# pair tile for the forward and dZ GEMMs (K = H), per pair tile and 64-column
-# K block for the dX GEMM (K = the vocabulary, split or not). A bench launch's
-# traffic is that figure times its units. Valid while the GEMM sources hash to
-# `sha` (otherwise the line reports traffic as null); the paired dW GEMM's
-# traffic is not proportional to its units and is not estimated.
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of each GEMM kind,
+# the mean over every launch of one bench step of `workload` (dW paired, the
+# logits recomputed: the headline leg), from one ncu capture of those launches
+# (a one-pass metric set, caches cold before each launch). Valid for that
+# workload while the GEMM sources hash to `sha`; otherwise the line reports
+# traffic as null.
 TRAFFIC = {
-    "sha": "b09fe802cf16f4b1a53e8110949a5cacfcfd7b4efa625a9cef3bd6e203b4d2cc",
-    "bytes_per_tile": {"lmhead_fwd_lse": 1.82e5, "lmhead_dz": 3.49e5},
-    "bytes_per_tile_kblock": {"dx_gemm": 1.35e4},
-    "source": "llada8b_r512_b8 small case, samples 12-13 (M = 3209, 3423), scaled by units",
+    "sha": "53ba1dffebd400f05cb22f497db35ca8a8f5ea789bba2b3b761438bc725e03c8",
+    "workload": "llada8b_r512_onpolicy",
+    "bytes_per_launch": {"lmhead_fwd_lse": 1.858e9, "lmhead_dz": 3.691e9, "dx_gemm": 3.743e9,
+                         "dw_gemm": 13.095e9},
+    "source": "ncu over the 168 launches of one bench step (llada8b_r512_onpolicy, dW paired), "
+              "mean per launch",
 }
 
 
@@ -411,13 +411,9 @@ def main():
         dom_avg_s = dom_ms / dom_launches / 1e3
         achieved = dom_flops_per_launch / dom_avg_s / 1e12
         traffic = None
-        if headline_mode and TRAFFIC["sha"] == kernel_sha():
-            row_blocks = sum(-(-m // 256) for m in rows_per_sample) / n_t   # per launch
-            if dom in TRAFFIC["bytes_per_tile"]:
-                traffic = TRAFFIC["bytes_per_tile"][dom] * row_blocks * (-(-V // 256))
-            elif dom in TRAFFIC["bytes_per_tile_kblock"]:
-                traffic = (TRAFFIC["bytes_per_tile_kblock"][dom] * row_blocks * (-(-H // 256))
-                           * (-(-V // 64)))
+        if (headline_mode and args.workload == TRAFFIC["workload"] and world == 1
+                and TRAFFIC["sha"] == kernel_sha()):
+            traffic = TRAFFIC["bytes_per_launch"].get(dom)
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sustained"], "traffic": traffic,
                 "traffic_source": TRAFFIC["source"] if traffic is not None else None,
