@@ -80,6 +80,36 @@ BGPO_HD int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 // Column tiles of the dX GEMM for `tiles_h` hidden-size blocks of kBN columns.
 BGPO_HD int64_t dx_tiles_n(int64_t tiles_h) { return ceil_div(tiles_h, kDxWide); }
 
+// Row groups of the forward and dZ GEMMs. Consecutive tiles share a vocabulary
+// tile of W, so every wave of tiles reads all of Xm's row blocks; once Xm
+// outgrows what L2 keeps from one wave to the next (measured at the 8B head:
+// no re-reads up to 36 MB, 3.5-5 reads per launch at 56-64 MB), the row blocks
+// are walked in groups of at most kXmGroupBytes of Xm, each group over the
+// whole vocabulary: W is then read once per group instead of Xm once per wave.
+constexpr int64_t kXmGroupMinBytes = int64_t(52) << 20;
+constexpr int64_t kXmGroupBytes = int64_t(40) << 20;
+BGPO_HD int64_t xm_row_groups(int64_t tiles_m, int64_t H) {
+  const int64_t bytes = tiles_m * kPairM * H * 2;
+  if (tiles_m <= 1 || bytes <= kXmGroupMinBytes) return 1;
+  const int64_t g = ceil_div(bytes, kXmGroupBytes);
+  return g < tiles_m ? g : tiles_m;
+}
+
+// Tile (row block, vocabulary tile) of unit u of the forward and dZ GEMMs with
+// `groups` row groups: group g holds row blocks [g tm / G, (g + 1) tm / G),
+// its units follow those of the groups before it, and consecutive units of a
+// group share a vocabulary tile.
+BGPO_HD void row_group_tile(int64_t u, int64_t tiles_m, int64_t tiles_n, int64_t groups,
+                            int64_t* m_blk, int64_t* n_blk) {
+  int64_t g = 0;
+  while (g + 1 < groups && ((g + 1) * tiles_m / groups) * tiles_n <= u) ++g;
+  const int64_t r0 = g * tiles_m / groups;
+  const int64_t rows = (g + 1) * tiles_m / groups - r0;
+  const int64_t local = u - r0 * tiles_n;
+  *n_blk = local / rows;
+  *m_blk = r0 + local % rows;
+}
+
 // Split-K count of the dX GEMM (K = vocabulary) for `mb` pair row blocks times
 // `tiles_n` column tiles on `num_pairs` CTA pairs: the smallest s whose
 // wave-quantised time ceil(tiles*s/pairs)/s is within 8% of the ideal

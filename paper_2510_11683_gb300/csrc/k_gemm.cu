@@ -72,6 +72,7 @@ struct GemmParams {
 struct Work {
   int64_t units, tiles_m, tiles_n, kb_total;
   int64_t kb_first;  // first K block (dW: a partner already added is skipped)
+  int64_t groups;    // forward and dZ: row groups (xm_row_groups)
   int splits;
 };
 
@@ -88,12 +89,14 @@ __device__ __forceinline__ Work make_work(const GemmParams& p, int32_t M, int64_
   Work w;
   w.splits = 1;
   w.kb_first = 0;
+  w.groups = 1;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
     w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = KIND == GEMM_FWD ? p.g.n_vt : ceil_div(p.v_end - p.v_begin, kBN);
     // a last K block past H reads the tensor maps' zero fill
     w.kb_total = ceil_div(p.g.H, kBK);
     w.units = w.tiles_m * w.tiles_n;
+    w.groups = xm_row_groups(w.tiles_m, p.g.H);
   } else if (KIND == GEMM_DX) {
     w.tiles_m = ceil_div(M, kPairM);
     w.tiles_n = dx_tiles_n(p.g.tiles_h);
@@ -120,8 +123,11 @@ __device__ __forceinline__ Unit unit_of(const Work& w, int64_t u) {
   t.split = 0;
   if (KIND == GEMM_FWD || KIND == GEMM_DZ) {
     // consecutive units share a vocabulary tile of W: it is read from HBM once
-    t.n_blk = (int32_t)(u / w.tiles_m);
-    t.m_blk = (int32_t)(u % w.tiles_m);
+    // per row group
+    int64_t m, n;
+    row_group_tile(u, w.tiles_m, w.tiles_n, w.groups, &m, &n);
+    t.m_blk = (int32_t)m;
+    t.n_blk = (int32_t)n;
     t.kb0 = 0;
     t.kb_n = (int32_t)w.kb_total;
   } else if (KIND == GEMM_DX) {

@@ -68,6 +68,27 @@ int main() {
   for (const auto& s : shapes) layout(s[0], s[1], s[2], s[3]);
   for (int32_t j : {0, 1, 2, 15, 16, 1000, 65534, 65535})
     printf("{\"kind\": \"tag\", \"j\": %d, \"tag\": %d}\n", j, pend_tag(j));
+  // row groups of the forward / dZ GEMMs: every tile exactly once
+  for (int64_t H : {64, 3584, 4096, 16384})
+    for (int64_t tm : {1, 2, 3, 17, 25, 26, 28, 32, 64, 129})
+      for (int64_t tn : {1, 7, 494}) {
+        const int64_t G = xm_row_groups(tm, H);
+        static int seen[129 * 494];
+        for (int64_t i = 0; i < tm * tn; ++i) seen[i] = 0;
+        long long bad = 0, prev_n = -1, runs = 0;
+        for (int64_t u = 0; u < tm * tn; ++u) {
+          int64_t m, n;
+          row_group_tile(u, tm, tn, G, &m, &n);
+          if (m < 0 || m >= tm || n < 0 || n >= tn) { ++bad; continue; }
+          ++seen[m * tn + n];
+          if (n != prev_n) { ++runs; prev_n = n; }
+        }
+        long long once = 0;
+        for (int64_t i = 0; i < tm * tn; ++i) once += seen[i] == 1;
+        printf("{\"kind\": \"group\", \"H\": %lld, \"tm\": %lld, \"tn\": %lld, \"G\": %lld, "
+               "\"bad\": %lld, \"once\": %lld, \"runs\": %lld}\n",
+               (long long)H, (long long)tm, (long long)tn, (long long)G, bad, once, runs);
+      }
   return 0;
 }
 """
@@ -85,7 +106,7 @@ def plan(tmp_path_factory):
     subprocess.run([cxx, "-std=c++17", "-O1", "-I", CSRC, str(src), "-o", str(exe)], check=True)
     out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout
     recs = [json.loads(line) for line in out.splitlines()]
-    return {k: [r for r in recs if r["kind"] == k] for k in ("layout", "split", "roff", "tag")}
+    return {k: [r for r in recs if r["kind"] == k] for k in ("layout", "split", "roff", "tag", "group")}
 
 
 def _ceil(a, b):
@@ -202,3 +223,17 @@ def test_vocabulary_chunks(plan):
         assert L["local"] == int(L["n_vc"] > 1 and not L["pair"])
         assert L["dz_cols"] == (vc if L["local"] else v_pad)
         assert vc % 256 == 0 or vc == v_pad
+
+
+def test_row_groups_cover_every_tile_once(plan):
+    for r in plan["group"]:
+        tm, tn, G, H = r["tm"], r["tn"], r["G"], r["H"]
+        assert r["bad"] == 0 and r["once"] == tm * tn, r
+        xm = tm * 256 * H * 2
+        if xm <= 52 << 20 or tm == 1:
+            assert G == 1, r
+        else:
+            # groups of at most 40 MB of Xm, never more groups than row blocks
+            assert G == min(tm, _ceil(xm, 40 << 20)), r
+        # a vocabulary tile's units are consecutive within each group
+        assert r["runs"] == G * tn or tn == 1, r
