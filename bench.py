@@ -53,11 +53,11 @@ UNIT = "tokens/s"
 # workload while the GEMM sources hash to `sha`; otherwise the line reports
 # traffic as null.
 TRAFFIC = {
-    "sha": "53ba1dffebd400f05cb22f497db35ca8a8f5ea789bba2b3b761438bc725e03c8",
+    "sha": "981f980e3a7dad317219b89f4aa070d106cc6dba692a8370f6e7e2c06829d45a",
     "workload": "llada8b_r512_onpolicy",
-    "bytes_per_launch": {"lmhead_fwd_lse": 1.858e9, "lmhead_dz": 3.691e9, "dx_gemm": 3.743e9,
-                         "dw_gemm": 13.095e9},
-    "source": "ncu over the 168 launches of one bench step (llada8b_r512_onpolicy, dW paired), "
+    "bytes_per_launch": {"lmhead_fwd_lse": 1.561e9, "lmhead_dz": 3.275e9, "dx_gemm": 4.363e9,
+                         "dw_gemm": 14.406e9},
+    "source": "ncu over the 56 GEMM launches of one bench step (llada8b_r512_onpolicy, dW paired), "
               "mean per launch",
 }
 
