@@ -507,18 +507,43 @@ def test_peak_device_memory_flat_in_n_t(bg, pair):
     assert peaks[16] - peaks[1] <= vectors + (1 << 20), peaks
 
 
-@pytest.mark.parametrize("H", [72, 200, 328])
+@pytest.mark.parametrize("H", [72, 200, 328, 768, 1000])
 def test_hidden_sizes_not_a_multiple_of_64(bg, H):
     """H a multiple of 8 only: the forward and dZ GEMMs end on a partial K
     block (read as zeros), the dX and dW GEMMs on a partial hidden-size tile
     and 32-column sub-tile (8 columns of H = 200, 72 and 328), the transpose
     on a partial 64-column tile; with and without vocabulary chunks and dW
-    pairing."""
+    pairing. The dX GEMM's tiles are two 256-column blocks of H wide: H = 768
+    has an odd number of blocks (the last tile's second block lies wholly past
+    H), H = 1000 ends inside the last tile's second block."""
     wl = CONFIGS["ragged"].with_(name="odd_hidden", H=H, seed=90 + H)
     inp_cpu = make_inputs(wl)
     inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
     o = oracle_run(wl, inp_cpu)
     for kw in (dict(), dict(vocab_chunk=256), dict(pair_dw=True), dict(keep_logits=True)):
+        g = gpu_run(wl, inp, **kw)
+        assert bg.get_device_error(g["ws"]) == (0, 0), kw
+        assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
+        assert rel_ell_err(to64(g["ell"]), o["ell"]).max() <= ELL_TOL, kw
+        assert normwise(to64(g["dX"]), o["dX"]) <= GRAD_TOL, kw
+        assert normwise(to64(g["dW"]), o["dW"]) <= GRAD_TOL, kw
+
+
+def test_row_groups_of_the_forward_and_dz_gemms(bg):
+    """H = 16384, so that a sample of about 3,000 masked rows holds about
+    100 MB of gathered rows Xm: the forward and dZ GEMMs walk its row blocks in
+    groups (more than 52 MB of Xm: groups of at most 40 MB), the other sample
+    stays in one group. Every l, all of dX and dW against the oracle, with the
+    default flags, dW pairing and kept logits."""
+    wl = CONFIGS["ragged_strat"].with_(name="row_groups", B=4, P=3, R=1001, H=16384, V=1000,
+                                       n_t=2, G=4, seed=77)
+    inp_cpu = make_inputs(wl)
+    inp = {k: (v.cuda() if v is not None else None) for k, v in inp_cpu.items()}
+    o = oracle_run(wl, inp_cpu)
+    rows = o["masks"].reshape(wl.n_t, -1).sum(axis=1)
+    xm_bytes = [-(-int(m) // 256) * 256 * wl.H * 2 for m in rows]
+    assert max(xm_bytes) > 52 << 20 >= min(xm_bytes), rows    # grouped and ungrouped samples
+    for kw in (dict(), dict(pair_dw=True), dict(keep_logits=True)):
         g = gpu_run(wl, inp, **kw)
         assert bg.get_device_error(g["ws"]) == (0, 0), kw
         assert np.array_equal(g["masks"].cpu().numpy(), o["masks"])
