@@ -31,9 +31,10 @@ __device__ __forceinline__ int32_t rows_of_sample(int32_t* err, int32_t j, int32
 
 // ---------------------------------------------------------------------------
 // Forward masking process (Sec. 2.1; Eq. 3, 5) + stable compaction.
-// One CTA of 1024 threads walks the (b, q) Philox blocks in ascending order,
-// 1024 blocks per round; a block-wide exclusive scan places every masked
-// position (b, i) at its rank, so rows[] is sorted by b * R + i.
+// One CTA of 1024 threads first draws every sequence's t (one Philox block
+// each, kept in the workspace), then walks the (b, q) mask blocks in ascending
+// order, 1024 blocks per round; a block-wide exclusive scan places every
+// masked position (b, i) at its rank, so rows[] is sorted by b * R + i.
 // ---------------------------------------------------------------------------
 constexpr int kScanThreads = 1024;
 
@@ -45,7 +46,19 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
   const int64_t nblk = (int64_t)a.B * Q;
   const uint64_t d_over_2_24 = (a.t_mode == 1) ? (uint64_t)a.n_t : 1ull;   // D / 2^24
   if (tid == 0) s_carry = 0;
-  __syncthreads();
+  // t of every sequence: T = u24 + 1 (i.i.d.) or j 2^24 + u24 + 1 (stratified)
+  for (int32_t b = tid; b < a.B; b += kScanThreads) {
+    const uint64_t bg = (uint64_t)b + (uint64_t)a.b_offset;   // global sequence index
+    const PhiloxOut ot = philox4x64_10(0, bg, (uint64_t)a.j, kStreamT, a.seed, 0);
+    const uint64_t u = ot.w[0] >> kU24Shift;
+    const uint64_t T = (a.t_mode == 1) ? ((uint64_t)a.j << 24) + u + 1 : u + 1;
+    const float tf = (float)((double)T / (double)(d_over_2_24 << 24));
+    w.t[b] = tf;
+    w.tnum[2 * b] = (uint32_t)T;
+    w.tnum[2 * b + 1] = (uint32_t)(T >> 32);
+    if (a.t_out) a.t_out[b] = tf;
+  }
+  __syncthreads();  // the block's T values are visible to every thread
   for (int64_t base = 0; base < nblk; base += kScanThreads) {
     const int64_t e = base + tid;
     int32_t cnt = 0;
@@ -56,9 +69,7 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
       q = (int32_t)(e % Q);
       const uint64_t bg = (uint64_t)b + (uint64_t)a.b_offset;   // global sequence index
       const int32_t len = a.resp_len ? min(max(a.resp_len[b], 0), a.R) : a.R;
-      const PhiloxOut ot = philox4x64_10(0, bg, (uint64_t)a.j, kStreamT, a.seed, 0);
-      const uint64_t u = ot.w[0] >> kU24Shift;
-      const uint64_t T = (a.t_mode == 1) ? ((uint64_t)a.j << 24) + u + 1 : u + 1;
+      const uint64_t T = (uint64_t)w.tnum[2 * b] | ((uint64_t)w.tnum[2 * b + 1] << 32);
       const PhiloxOut om = philox4x64_10((uint64_t)q, bg, (uint64_t)a.j, kStreamMask, a.seed, 0);
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
@@ -71,13 +82,6 @@ __global__ void __launch_bounds__(kScanThreads) k_mask_compact(MaskArgs a, WsPtr
           cnt += (int32_t)bit;
           if (a.mask_out) a.mask_out[(int64_t)b * a.R + i] = (uint8_t)bit;
         }
-      }
-      if (q == 0) {
-        const float tf = (float)((double)T / (double)(d_over_2_24 << 24));
-        w.t[b] = tf;
-        w.tnum[2 * b] = (uint32_t)T;
-        w.tnum[2 * b + 1] = (uint32_t)(T >> 32);
-        if (a.t_out) a.t_out[b] = tf;
       }
     }
     // block-wide exclusive scan of cnt
@@ -398,10 +402,15 @@ __global__ void k_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const fl
 // ---------------------------------------------------------------------------
 // dX[b, i, :] += sum_s partial_s[r, :] over the split-K partials of the dX GEMM
 // (fixed split order; rows are unique within a sample, so no atomics). With a
-// single split the GEMM's epilogue has already added its tile into dX.
+// single split the GEMM's epilogue has already added its tile into dX. Each
+// thread keeps kDxrVec 16-byte loads of a split (and of the dX row) in flight
+// at once.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs w,
-                                                   float* __restrict__ dX) {
+constexpr int kDxrThreads = 256;
+constexpr int kDxrVec = 4;
+
+__global__ void __launch_bounds__(kDxrThreads) k_dx_reduce(Geometry g, int32_t j, WsPtrs w,
+                                                           float* __restrict__ dX) {
   const int32_t M = rows_of_sample(w.err, j, KID_DX_REDUCE);
   const int64_t r = blockIdx.x;
   if (r >= M) return;
@@ -415,17 +424,38 @@ __global__ void __launch_bounds__(256) k_dx_reduce(Geometry g, int32_t j, WsPtrs
   const int64_t split_stride = mb * kPairM * g.H / 4;
   const int32_t idx = w.rows[r];
   if (!BGPO_IN_BOUNDS(w.err, idx >= 0 && idx < g.m_cap, KID_DX_REDUCE * 16 + 9)) return;
-  const float4* src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
+  const float4* __restrict__ src = reinterpret_cast<const float4*>(w.dxp) + r * (g.H / 4);
   float4* dst = reinterpret_cast<float4*>(dX) + (int64_t)idx * (g.H / 4);
-  for (int64_t h = threadIdx.x; h < g.H / 4; h += blockDim.x) {
-    float4 acc = src[h];
-    for (int s = 1; s < S; ++s) {
-      const float4 v = src[s * split_stride + h];
-      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+  const int64_t nvec = g.H / 4;
+  for (int64_t h0 = threadIdx.x; h0 < nvec; h0 += (int64_t)kDxrThreads * kDxrVec) {
+    float4 acc[kDxrVec], o[kDxrVec];
+#pragma unroll
+    for (int k = 0; k < kDxrVec; ++k) {
+      const int64_t h = h0 + (int64_t)k * kDxrThreads;
+      const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+      acc[k] = h < nvec ? src[h] : z;
+      o[k] = h < nvec ? dst[h] : z;
     }
-    float4 o = dst[h];
-    o.x += acc.x; o.y += acc.y; o.z += acc.z; o.w += acc.w;
-    dst[h] = o;
+    for (int s = 1; s < S; ++s) {
+      float4 v[kDxrVec];
+#pragma unroll
+      for (int k = 0; k < kDxrVec; ++k) {
+        const int64_t h = h0 + (int64_t)k * kDxrThreads;
+        v[k] = h < nvec ? src[s * split_stride + h] : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < kDxrVec; ++k) {
+        acc[k].x += v[k].x; acc[k].y += v[k].y; acc[k].z += v[k].z; acc[k].w += v[k].w;
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kDxrVec; ++k) {
+      const int64_t h = h0 + (int64_t)k * kDxrThreads;
+      if (h < nvec) {
+        o[k].x += acc[k].x; o[k].y += acc[k].y; o[k].z += acc[k].z; o[k].w += acc[k].w;
+        dst[h] = o[k];
+      }
+    }
   }
 }
 
@@ -622,7 +652,7 @@ cudaError_t launch_vrpo_coeffs(int32_t B, int32_t n_t, float loss_scale, const f
 
 cudaError_t launch_dx_reduce(const Geometry& g, int32_t j, const WsPtrs& w, float* dX,
                              cudaStream_t s) {
-  k_dx_reduce<<<(unsigned)g.m_cap, 256, 0, s>>>(g, j, w, dX);
+  k_dx_reduce<<<(unsigned)g.m_cap, kDxrThreads, 0, s>>>(g, j, w, dX);
   return cudaGetLastError();
 }
 
