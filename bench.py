@@ -227,13 +227,22 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
+L2_BYTES = 129e6
+
+
 def config_of(wl):
-    return {"workload": f"{wl.name}: LLaDA-8B-shaped LM head H={wl.H} V={wl.V}, {wl.B} responses "
+    head = {(4096, 126464): "LLaDA-8B-shaped LM head",
+            (3584, 152064): "Dream-7B-shaped LM head"}.get((wl.H, wl.V), "LM head")
+    w_bytes = 2.0 * wl.H * wl.V
+    l2 = (f"inputs larger than L2 (W alone is {w_bytes / 1e9:.2f} GB > 129 MB); no flush"
+          if w_bytes > L2_BYTES else
+          f"inputs fit in L2 (W is {w_bytes / 1e6:.2f} MB); no flush: a launch-bound case")
+    return {"workload": f"{wl.name}: {head} H={wl.H} V={wl.V}, {wl.B} responses "
                         f"x (prompt {wl.P} + response {wl.R}), n_t={wl.n_t} "
                         f"{'stratified' if wl.t_mode else 'iid'} t, G={wl.G}, "
                         f"{'on-policy' if wl.eps_std == 0 else 'off-policy'}",
             "B": wl.B, "P": wl.P, "R": wl.R, "H": wl.H, "V": wl.V, "n_t": wl.n_t, "G": wl.G,
-            "l2": "inputs larger than L2 (W alone is 1.04 GB > 129 MB); no flush"}
+            "l2": l2}
 
 
 # ----------------------------------------------------------------------------------
