@@ -261,3 +261,41 @@ def test_kept_and_recomputed_logit_chunks_agree(monkeypatch):
     again = O.elbo_term_grads(X, W, Y, P, masks[1], ts[1], coef, chunk=6, with_ell=True)
     for a, b in zip(kept, again):
         assert np.allclose(a, b, rtol=1e-14, atol=1e-15)
+
+
+def test_brute_force_gradient_unbiased_over_all_masks():
+    # Sec. 2.1 / Eq. 3-4, differentiated: with every response token masked
+    # independently with probability t, the mask-weighted mean of the one-sample
+    # gradient of l (its 1/t weight included) is the gradient of
+    # sum_i log p(y^i | x) over all response positions, for every t. The right
+    # side is torch autograd on log_softmax, independent of the oracle.
+    import itertools
+    rng = np.random.default_rng(31)
+    B, P, R, H, V = 2, 2, 8, 6, 12
+    X = rng.standard_normal((B, P + R, H)) * 1.3
+    W = rng.standard_normal((V, H)) * 0.8
+    Y = rng.integers(0, V, size=(B, R))
+    Xt = torch.from_numpy(X.copy()).requires_grad_(True)
+    Wt = torch.from_numpy(W.copy()).requires_grad_(True)
+    total = 0
+    for b in range(B):
+        z = Xt[b, P:] @ Wt.T
+        total = total + torch.log_softmax(z, dim=1).gather(1, torch.from_numpy(Y[b])[:, None]).sum()
+    total.backward()
+    gX = Xt.grad.numpy()[:, P:]
+    gW = Wt.grad.numpy()
+    coef = np.ones(B)
+    for t in (0.2, 0.55, 1.0):
+        aX = np.zeros((B, R, H))
+        aW = np.zeros((V, H))
+        for bits in itertools.product((0, 1), repeat=R):
+            m = np.array(bits, dtype=np.uint8)
+            k = int(m.sum())
+            weight = t ** k * (1 - t) ** (R - k)
+            if weight == 0.0:
+                continue
+            dX, dW = O.elbo_term_grads(X, W, Y, P, np.stack([m] * B), np.full(B, t), coef)
+            aX += weight * dX
+            aW += weight * dW
+        assert np.allclose(aX, gX, rtol=1e-10, atol=1e-12)
+        assert np.allclose(aW, gW, rtol=1e-10, atol=1e-12)
